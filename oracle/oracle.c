@@ -242,7 +242,7 @@ int64_t or_int_range_map32(int64_t lo, uint64_t r, uint32_t w) {
 /* Values >= N are walked again through the same map until they land in     */
 /* [0, N) (cycle walking), which keeps the map a bijection of [0, N).        */
 uint64_t or_perm_value(uint64_t N, uint64_t seed, uint32_t stream, uint64_t g) {
-  if (N <= 1) return 0;
+  if (N <= 1 || g >= N) return 0; /* defined on [0, N) only */
   int k = 0;
   while (k < 64 && ((uint64_t)1 << k) < N) ++k;
   uint64_t mask = (k >= 64) ? ~(uint64_t)0 : (((uint64_t)1 << k) - 1);

@@ -1,0 +1,295 @@
+"""Python binding of libsynverify (include/synverify.h): argument marshalling only.
+
+GB300 (sm_103a) implementation of the data-parallel path of Synthesis-Based
+Verification (CUDA-Harness, Sec. 4.2):
+
+  generate(specs, arena)            syn_generate: seeded test-data synthesis
+  compare(pairs, cand, ref)         verify_compare: Eq. 1 per segment
+  progressive(stages, cand, ref)    verify_progressive: fail-fast stage ladder
+
+Device memory and streams come from PyTorch (tensors are passed by
+data_ptr(); the current CUDA stream is used unless one is given).  Every step
+of the path runs in the library's CUDA kernels; there is no CPU fallback: if
+the compiled library is missing, importing works but every call raises.
+
+Specs and pairs are any objects with the attribute names of `GenSpec`,
+`Perturb` and `Pair` below (string-valued enums).
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from dataclasses import dataclass, field
+from typing import List, Optional, Sequence, Tuple
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "_build", "libsynverify.so")
+
+DTYPES = {"f32": 0, "f16": 1, "bf16": 2, "i32": 3, "i64": 4, "u32": 5}
+DTYPE_BYTES = {"f32": 4, "f16": 2, "bf16": 2, "i32": 4, "i64": 8, "u32": 4}
+DISTS = {"uniform": 0, "normal": 1, "int_range": 2, "permutation": 3, "dotlike": 4, "raw_bits": 5,
+         "constant": 6}
+SPECIALS = {"nan": 1, "pinf": 2, "ninf": 4, "denorm": 8, "zero": 16, "imin": 32, "imax": 64, "dup": 128}
+PERTS = {"none": 0, "rate_add_pm": 1, "rel_noise": 2, "count_set": 3, "count_add": 4, "swap_pairs": 5}
+EQUAL_NAN = 1
+STAGE_RUN, STAGE_SKIPPED = 1, 2
+NO_OUTPUT = (1 << 64) - 1
+INLINE_ENTRIES = 8
+STATUS = {0: "SV_OK", -1: "SV_EINVAL", -2: "SV_EALIGN", -3: "SV_ERANGE", -4: "SV_EWORKSPACE", -5: "SV_ECUDA"}
+
+
+# ---------------------------------------------------------------------------
+# public spec types (mirrors of the C structs with string enums)
+# ---------------------------------------------------------------------------
+@dataclass
+class Perturb:
+    kind: str = "none"
+    stream: int = 0
+    rate: float = 0.0
+    count: int = 0
+    value: float = 0.0
+    ivalue: int = 0
+
+
+@dataclass
+class GenSpec:
+    dtype: str
+    dist: str
+    n: int
+    seed: int = 0
+    stream: int = 0
+    ref_offset: Optional[int] = None
+    cand_offset: Optional[int] = None
+    elem_offset: int = 0
+    logical_n: int = 0
+    p0: float = 0.0
+    p1: float = 0.0
+    i0: int = 0
+    i1: int = 0
+    specials: Tuple[str, ...] = ()
+    special_rate: float = 0.0
+    rows: int = 0
+    cols: int = 0
+    dot_k: int = 0
+    a_offset: int = 0
+    b_offset: int = 0
+    pelem: Perturb = field(default_factory=Perturb)
+    pcount: Perturb = field(default_factory=Perturb)
+
+
+@dataclass
+class Pair:
+    dtype: str
+    n: int
+    cand_offset: int
+    ref_offset: int
+    atol: float = 0.0
+    rtol: float = 0.0
+    equal_nan: bool = True
+
+
+# ---------------------------------------------------------------------------
+# C structs (layouts of synverify.h)
+# ---------------------------------------------------------------------------
+class sv_perturb(C.Structure):
+    _fields_ = [("kind", C.c_uint32), ("stream", C.c_uint32), ("rate", C.c_double), ("count", C.c_uint64),
+                ("value", C.c_double), ("ivalue", C.c_int64)]
+
+
+class syn_spec(C.Structure):
+    _fields_ = [("dtype", C.c_uint32), ("dist", C.c_uint32), ("n", C.c_uint64), ("seed", C.c_uint64),
+                ("stream", C.c_uint32), ("special_mask", C.c_uint32), ("special_rate", C.c_double),
+                ("ref_offset", C.c_uint64), ("cand_offset", C.c_uint64), ("elem_offset", C.c_uint64),
+                ("logical_n", C.c_uint64), ("p0", C.c_double), ("p1", C.c_double), ("i0", C.c_int64),
+                ("i1", C.c_int64), ("rows", C.c_uint64), ("cols", C.c_uint64), ("dot_k", C.c_uint64),
+                ("a_offset", C.c_uint64), ("b_offset", C.c_uint64), ("pelem", sv_perturb), ("pcount", sv_perturb)]
+
+
+class vc_pair(C.Structure):
+    _fields_ = [("dtype", C.c_uint32), ("flags", C.c_uint32), ("n", C.c_uint64), ("cand_offset", C.c_uint64),
+                ("ref_offset", C.c_uint64), ("atol", C.c_double), ("rtol", C.c_double)]
+
+
+class vc_result(C.Structure):
+    _fields_ = [("mismatches", C.c_uint64), ("nan_disagree", C.c_uint64), ("inf_disagree", C.c_uint64),
+                ("n_finite", C.c_uint64), ("first_mismatch", C.c_int64), ("max_abs_u64", C.c_uint64),
+                ("max_abs", C.c_double), ("max_rel", C.c_double), ("rms", C.c_double), ("pass_", C.c_uint32),
+                ("state", C.c_uint32)]
+
+
+assert C.sizeof(syn_spec) == 224 and C.sizeof(vc_pair) == 48 and C.sizeof(vc_result) == 80
+RESULT_BYTES = C.sizeof(vc_result)
+
+# every function the header declares: (name, restype, argtypes)
+_VP, _SZ = C.c_void_p, C.c_size_t
+EXPORTS = [
+    ("sv_generate_workspace_bytes", _SZ, [C.POINTER(syn_spec), C.c_int]),
+    ("sv_compare_workspace_bytes", _SZ, [C.POINTER(vc_pair), C.c_int]),
+    ("sv_progressive_workspace_bytes", _SZ, [C.POINTER(vc_pair), C.c_int]),
+    ("sv_check_specs", C.c_int, [C.POINTER(syn_spec), C.c_int, _SZ]),
+    ("sv_check_pairs", C.c_int, [C.POINTER(vc_pair), C.c_int, _SZ, _SZ]),
+    ("syn_generate", C.c_int, [C.POINTER(syn_spec), C.c_int, _VP, _SZ, _VP, _SZ, _VP]),
+    ("verify_compare", C.c_int, [C.POINTER(vc_pair), C.c_int, _VP, _SZ, _VP, _SZ, _VP, _VP, _SZ, _VP]),
+    ("verify_progressive", C.c_int, [C.POINTER(vc_pair), C.c_int, _VP, _SZ, _VP, _SZ, _VP, _VP, _VP, _SZ, _VP]),
+    ("sv_strerror", C.c_char_p, [C.c_int]),
+    ("sv_abi_version", C.c_int, []),
+]
+
+_lib = None
+
+
+def lib() -> C.CDLL:
+    """The loaded library; raises if it has not been built (no fallback)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError("libsynverify.so is not built (%s); run __graft_entry__.build() or "
+                               "python -m paper_2609_00058_gb300.build" % LIB_PATH)
+        L = C.CDLL(LIB_PATH)
+        for name, res, args in EXPORTS:
+            f = getattr(L, name)
+            f.restype, f.argtypes = res, args
+        _lib = L
+    return _lib
+
+
+class SynVerifyError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        msg = lib().sv_strerror(status).decode()
+        super().__init__("%s failed: %s (%s)" % (where, STATUS.get(status, status), msg))
+        self.status = status
+
+
+def _ok(status: int, where: str) -> None:
+    if status != 0:
+        raise SynVerifyError(status, where)
+
+
+# ---------------------------------------------------------------------------
+# marshalling
+# ---------------------------------------------------------------------------
+def _perturb(p) -> sv_perturb:
+    return sv_perturb(PERTS[p.kind], p.stream, p.rate, p.count, p.value, p.ivalue)
+
+
+def to_c_spec(s) -> syn_spec:
+    mask = 0
+    for k in s.specials:
+        mask |= SPECIALS[k]
+    return syn_spec(DTYPES[s.dtype], DISTS[s.dist], s.n, s.seed, s.stream, mask, s.special_rate,
+                    NO_OUTPUT if s.ref_offset is None else s.ref_offset,
+                    NO_OUTPUT if s.cand_offset is None else s.cand_offset,
+                    s.elem_offset, s.logical_n, s.p0, s.p1, s.i0, s.i1, s.rows, s.cols, s.dot_k,
+                    s.a_offset, s.b_offset, _perturb(s.pelem), _perturb(s.pcount))
+
+
+def to_c_pair(p) -> vc_pair:
+    return vc_pair(DTYPES[p.dtype], EQUAL_NAN if p.equal_nan else 0, p.n, p.cand_offset, p.ref_offset,
+                   p.atol, p.rtol)
+
+
+class SpecTable:
+    """A prepared host table of generator specs (reusable across calls)."""
+
+    def __init__(self, specs: Sequence):
+        self.n = len(specs)
+        self.arr = (syn_spec * max(self.n, 1))(*[to_c_spec(s) for s in specs])
+        self.ws_bytes = lib().sv_generate_workspace_bytes(self.arr, self.n)
+
+
+class PairTable:
+    """A prepared host table of compare pairs / ladder stages."""
+
+    def __init__(self, pairs: Sequence, progressive: bool = False):
+        self.n = len(pairs)
+        self.arr = (vc_pair * max(self.n, 1))(*[to_c_pair(p) for p in pairs])
+        f = lib().sv_progressive_workspace_bytes if progressive else lib().sv_compare_workspace_bytes
+        self.ws_bytes = f(self.arr, self.n)
+
+
+def _stream_ptr(stream) -> int:
+    import torch
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _workspace(nbytes: int, device, workspace):
+    import torch
+    if nbytes == 0:
+        return None, 0
+    if workspace is not None:
+        return workspace.data_ptr(), workspace.numel() * workspace.element_size()
+    ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
+    base = ws.data_ptr()
+    off = (-base) % 256
+    return base + off, nbytes, ws  # keep the tensor alive
+
+
+def _nbytes(t) -> int:
+    return t.numel() * t.element_size()
+
+
+# ---------------------------------------------------------------------------
+# entry points
+# ---------------------------------------------------------------------------
+def generate(specs, arena, workspace=None, stream=None) -> None:
+    """syn_generate into `arena` (a CUDA tensor; offsets are bytes into it)."""
+    tab = specs if isinstance(specs, SpecTable) else SpecTable(specs)
+    ws = _workspace(tab.ws_bytes, arena.device, workspace)
+    rc = lib().syn_generate(tab.arr, tab.n, arena.data_ptr(), _nbytes(arena), ws[0], ws[1] if ws[0] else 0,
+                            _stream_ptr(stream))
+    _ok(rc, "syn_generate")
+
+
+def compare(pairs, cand, ref, results=None, workspace=None, stream=None):
+    """verify_compare; returns the device results tensor (uint8, n x 80 bytes)."""
+    import torch
+    tab = pairs if isinstance(pairs, PairTable) else PairTable(pairs)
+    if results is None:
+        results = torch.empty(max(tab.n, 1) * RESULT_BYTES, dtype=torch.uint8, device=cand.device)
+    ws = _workspace(tab.ws_bytes, cand.device, workspace)
+    rc = lib().verify_compare(tab.arr, tab.n, cand.data_ptr(), _nbytes(cand), ref.data_ptr(), _nbytes(ref),
+                              results.data_ptr(), ws[0], ws[1] if ws[0] else 0, _stream_ptr(stream))
+    _ok(rc, "verify_compare")
+    return results
+
+
+def progressive(stages, cand, ref, results=None, first_failed=None, workspace=None, stream=None):
+    """verify_progressive; returns (device results, device int32 first-failed index)."""
+    import torch
+    tab = stages if isinstance(stages, PairTable) else PairTable(stages, progressive=True)
+    if results is None:
+        results = torch.empty(max(tab.n, 1) * RESULT_BYTES, dtype=torch.uint8, device=cand.device)
+    if first_failed is None:
+        first_failed = torch.empty(1, dtype=torch.int32, device=cand.device)
+    ws = _workspace(tab.ws_bytes, cand.device, workspace)
+    rc = lib().verify_progressive(tab.arr, tab.n, cand.data_ptr(), _nbytes(cand), ref.data_ptr(), _nbytes(ref),
+                                  results.data_ptr(), first_failed.data_ptr(), ws[0], ws[1] if ws[0] else 0,
+                                  _stream_ptr(stream))
+    _ok(rc, "verify_progressive")
+    return results, first_failed
+
+
+def decode_results(results, n: int) -> List[dict]:
+    """Copy n vc_result records to the host as dicts."""
+    raw = bytes(results[: n * RESULT_BYTES].cpu().numpy().tobytes()) if hasattr(results, "cpu") else bytes(results)
+    out = []
+    for i in range(n):
+        r = vc_result.from_buffer_copy(raw, i * RESULT_BYTES)
+        out.append({"mismatches": r.mismatches, "nan_disagree": r.nan_disagree, "inf_disagree": r.inf_disagree,
+                    "n_finite": r.n_finite, "first_mismatch": r.first_mismatch, "max_abs_u64": r.max_abs_u64,
+                    "max_abs": r.max_abs, "max_rel": r.max_rel, "rms": r.rms, "pass": r.pass_, "state": r.state})
+    return out
+
+
+def check_specs(specs, arena_bytes: int) -> int:
+    tab = SpecTable(specs)
+    return lib().sv_check_specs(tab.arr, tab.n, arena_bytes)
+
+
+def check_pairs(pairs, cand_bytes: int, ref_bytes: int) -> int:
+    tab = PairTable(pairs)
+    return lib().sv_check_pairs(tab.arr, tab.n, cand_bytes, ref_bytes)

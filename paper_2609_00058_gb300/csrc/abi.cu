@@ -1,0 +1,384 @@
+// abi.cu -- the C ABI of synverify.h: host-side validation, workspace
+// layout, table upload and kernel launches.  No device memory is allocated
+// here; every device buffer comes from the caller.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <mutex>
+#include <vector>
+
+#include "sv_device.cuh"
+#include "sv_kernels.h"
+
+namespace sv {
+
+static_assert(sizeof(sv_perturb) == 40, "sv_perturb layout");
+static_assert(sizeof(syn_spec) == 224, "syn_spec layout");
+static_assert(sizeof(vc_pair) == 48, "vc_pair layout");
+static_assert(sizeof(vc_result) == 80, "vc_result layout");
+static_assert(sizeof(Partial) == 64, "partial record layout");
+static_assert(sizeof(DevSpec) == 240, "spec table entry layout");
+static_assert(sizeof(DevPair) == 80, "pair table entry layout");
+
+constexpr size_t kAlign = 256;
+static size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+// ---------------------------------------------------------------------------
+// per-device launch shape: one resident wave of each kernel, so every CTA of
+// a persistent grid runs at once and the contiguous chunks finish together
+// ---------------------------------------------------------------------------
+namespace {
+struct CapEntry {
+  int dev;
+  const void* fn;
+  uint32_t cap;
+};
+std::mutex g_mu;
+std::vector<CapEntry> g_caps;
+}  // namespace
+
+uint32_t grid_cap_for(const void* fn) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 152;
+  std::lock_guard<std::mutex> lk(g_mu);
+  for (const CapEntry& c : g_caps)
+    if (c.dev == dev && c.fn == fn) return c.cap;
+  int sms = 0, per_sm = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 152;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, 0) != cudaSuccess || per_sm <= 0)
+    per_sm = 1;
+  const uint32_t cap = (uint32_t)std::min<int>(sms * per_sm, (int)kGridCap);
+  g_caps.push_back(CapEntry{dev, fn, cap});
+  return cap;
+}
+
+LaunchShape shape_for(uint64_t tiles, uint32_t cap) {
+  LaunchShape s{0, 1};
+  if (tiles == 0) return s;
+  const uint64_t g = std::min<uint64_t>(tiles, std::max<uint32_t>(cap, 1));
+  s.chunk = (tiles + g - 1) / g;
+  s.grid = (uint32_t)((tiles + s.chunk - 1) / s.chunk);
+  return s;
+}
+
+// ---------------------------------------------------------------------------
+// validation
+// ---------------------------------------------------------------------------
+static bool add_ok(uint64_t a, uint64_t b, uint64_t limit) { return a <= limit && b <= limit - a; }
+
+static int check_range(uint64_t off, uint64_t bytes, uint64_t buf) {
+  if (off % 16) return SV_EALIGN;
+  if (!add_ok(off, bytes, buf)) return SV_ERANGE;
+  return SV_OK;
+}
+
+static bool valid_rate(double r) { return r >= 0.0 && r <= 1.0; }  // false for NaN
+
+static int check_spec(const syn_spec& s, uint64_t arena) {
+  if (s.dtype > SV_U32 || s.dist > SV_CONSTANT) return SV_EINVAL;
+  const bool fl = is_float((int)s.dtype);
+  switch (s.dist) {
+    case SV_UNIFORM: case SV_NORMAL: case SV_DOTLIKE: if (!fl) return SV_EINVAL; break;
+    case SV_INT_RANGE: case SV_PERMUTATION: if (fl) return SV_EINVAL; break;
+    default: break;
+  }
+  if (s.ref_offset == SV_NO_OUTPUT && s.cand_offset == SV_NO_OUTPUT) return SV_EINVAL;
+  if (s.elem_offset % 4) return SV_EALIGN;
+  if (!add_ok(s.elem_offset, s.n, SV_MAX_LOGICAL_N)) return SV_ERANGE;
+  const uint64_t N = s.logical_n ? s.logical_n : s.elem_offset + s.n;
+  if (N > SV_MAX_LOGICAL_N) return SV_ERANGE;
+  if (s.elem_offset + s.n > N) return SV_EINVAL;
+  const uint64_t bytes = s.n * elem_bytes((int)s.dtype);
+  int rc;
+  if (s.ref_offset != SV_NO_OUTPUT && (rc = check_range(s.ref_offset, bytes, arena))) return rc;
+  if (s.cand_offset != SV_NO_OUTPUT && (rc = check_range(s.cand_offset, bytes, arena))) return rc;
+  const uint32_t fmask = SV_SP_NAN | SV_SP_PINF | SV_SP_NINF | SV_SP_DENORM | SV_SP_ZERO | SV_SP_DUP;
+  const uint32_t imask = SV_SP_ZERO | SV_SP_IMIN | SV_SP_IMAX | SV_SP_DUP;
+  if (s.special_mask & ~(fl ? fmask : imask)) return SV_EINVAL;
+  if (!valid_rate(s.special_rate)) return SV_EINVAL;
+  if (s.dist == SV_UNIFORM && !(s.p1 >= s.p0)) return SV_EINVAL;
+  if (s.dist == SV_INT_RANGE) {
+    if (s.i1 < s.i0) return SV_EINVAL;
+    if (s.dtype == SV_I32 && (s.i0 < INT32_MIN || s.i1 > INT32_MAX)) return SV_EINVAL;
+    if (s.dtype == SV_U32 && (s.i0 < 0 || s.i1 > (int64_t)UINT32_MAX)) return SV_EINVAL;
+  }
+  if (s.dist == SV_PERMUTATION) {
+    if (s.dtype == SV_I32 && N > (1ull << 31)) return SV_ERANGE;
+    if (s.dtype == SV_U32 && N > (1ull << 32)) return SV_ERANGE;
+  }
+  if (s.dist == SV_DOTLIKE) {
+    if (s.cols == 0 || s.rows == 0 || s.cols % 4 || s.dot_k == 0 || s.dot_k > (1u << 20)) return SV_EINVAL;
+    if (s.rows > N / s.cols || s.rows * s.cols != N) return SV_EINVAL;
+    if (s.rows > (1ull << 40) / s.dot_k || s.cols > (1ull << 40) / s.dot_k) return SV_ERANGE;
+    if ((rc = check_range(s.a_offset, 4 * s.rows * s.dot_k, arena))) return rc;
+    if ((rc = check_range(s.b_offset, 4 * s.dot_k * s.cols, arena))) return rc;
+    if ((s.rows + 63) / 64 > 65535) return SV_ERANGE;  // grid.y of the tiled kernel
+  }
+  const sv_perturb& pe = s.pelem;
+  if (pe.kind != SV_PERT_NONE && pe.kind != SV_PERT_RATE_ADD_PM && pe.kind != SV_PERT_REL_NOISE) return SV_EINVAL;
+  if (pe.kind == SV_PERT_REL_NOISE && !fl) return SV_EINVAL;
+  if (pe.kind == SV_PERT_RATE_ADD_PM && !valid_rate(pe.rate)) return SV_EINVAL;
+  const sv_perturb& pc = s.pcount;
+  if (pc.kind != SV_PERT_NONE && pc.kind != SV_PERT_COUNT_SET && pc.kind != SV_PERT_COUNT_ADD &&
+      pc.kind != SV_PERT_SWAP_PAIRS)
+    return SV_EINVAL;
+  if (pc.kind != SV_PERT_NONE) {
+    if (pc.count == 0 || pc.count > SV_MAX_COUNT) return SV_EINVAL;
+    const uint64_t strata = pc.kind == SV_PERT_SWAP_PAIRS ? 2 * pc.count : pc.count;
+    if (strata > N) return SV_EINVAL;
+  }
+  return SV_OK;
+}
+
+static int check_pair(const vc_pair& p, uint64_t cand_bytes, uint64_t ref_bytes) {
+  if (p.dtype > SV_U32) return SV_EINVAL;
+  if (p.flags & ~(uint32_t)SV_EQUAL_NAN) return SV_EINVAL;
+  if (p.n > SV_MAX_LOGICAL_N) return SV_ERANGE;
+  if (is_float((int)p.dtype) && !(p.atol >= 0.0 && p.rtol >= 0.0)) return SV_EINVAL;  // NaN fails too
+  const uint64_t bytes = p.n * elem_bytes((int)p.dtype);
+  int rc;
+  if ((rc = check_range(p.cand_offset, bytes, cand_bytes))) return rc;
+  if ((rc = check_range(p.ref_offset, bytes, ref_bytes))) return rc;
+  return SV_OK;
+}
+
+static int check_specs(const syn_spec* specs, int n, size_t arena) {
+  if (n < 0 || n > SV_MAX_ENTRIES || (n > 0 && !specs)) return SV_EINVAL;
+  for (int i = 0; i < n; ++i)
+    if (int rc = check_spec(specs[i], arena)) return rc;
+  return SV_OK;
+}
+
+static int check_pairs(const vc_pair* pairs, int n, size_t cb, size_t rb) {
+  if (n < 0 || n > SV_MAX_ENTRIES || (n > 0 && !pairs)) return SV_EINVAL;
+  for (int i = 0; i < n; ++i)
+    if (int rc = check_pair(pairs[i], cb, rb)) return rc;
+  return SV_OK;
+}
+
+// ---------------------------------------------------------------------------
+// tables and workspace layout
+//   generate: [spec table, if n > SV_INLINE_ENTRIES]
+//   compare:  [pair table, if n > SV_INLINE_ENTRIES][partial slots]
+// Entries are stored grouped by kind (stable), one launch per group.
+// ---------------------------------------------------------------------------
+struct Group {
+  uint32_t key;
+  int begin, end;  // range in the grouped table
+  uint64_t tiles;
+  LaunchShape sh;
+};
+
+template <class KeyFn>
+static void group_by(int n, KeyFn key, std::vector<int>& order, std::vector<Group>& groups) {
+  order.resize(n);
+  for (int i = 0; i < n; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return key(a) < key(b); });
+  groups.clear();
+  for (int k = 0; k < n; ++k) {
+    if (groups.empty() || groups.back().key != key(order[k])) groups.push_back(Group{key(order[k]), k, k, 0, {0, 1}});
+    groups.back().end = k + 1;
+  }
+}
+
+static size_t spec_table_bytes(int n) { return n > SV_INLINE_ENTRIES ? align_up(sizeof(DevSpec) * (size_t)n) : 0; }
+static size_t pair_table_bytes(int n) { return n > SV_INLINE_ENTRIES ? align_up(sizeof(DevPair) * (size_t)n) : 0; }
+
+// partial slots of one group: CTA b of the group writes slot base + b + e for
+// its e-th pair, so a group needs grid + n - 1 slots; bounded without a device
+// by min(tiles, kGridCap) + n
+static size_t compare_partial_bytes(const vc_pair* pairs, int n) {
+  uint64_t tiles[8] = {0}, count[8] = {0};
+  for (int i = 0; i < n; ++i) {
+    tiles[pairs[i].dtype & 7] += cmp_tiles(pairs[i]);
+    count[pairs[i].dtype & 7] += 1;
+  }
+  uint64_t slots = 0;
+  for (int d = 0; d < 8; ++d)
+    if (count[d]) slots += std::min<uint64_t>(tiles[d], kGridCap) + count[d];
+  return align_up(sizeof(Partial) * (size_t)std::max<uint64_t>(slots, 1));
+}
+
+static int status_of(cudaError_t e) { return e == cudaSuccess ? SV_OK : SV_ECUDA; }
+
+static bool ws_ok(const void* ws, size_t have, size_t need) {
+  if (need == 0) return true;
+  return ws && have >= need && reinterpret_cast<uintptr_t>(ws) % kAlign == 0;
+}
+
+}  // namespace sv
+
+using namespace sv;
+
+extern "C" {
+
+int sv_abi_version(void) { return SV_ABI_VERSION; }
+
+const char* sv_strerror(int status) {
+  switch (status) {
+    case SV_OK: return "ok";
+    case SV_EINVAL: return "invalid argument (enum, count, tolerance, rate or dtype/dist pairing)";
+    case SV_EALIGN: return "misaligned offset (byte offsets must be multiples of 16, elem_offset of 4)";
+    case SV_ERANGE: return "data beyond its buffer, or a size beyond the library limits";
+    case SV_EWORKSPACE: return "workspace missing, misaligned or too small";
+    case SV_ECUDA: return "a CUDA launch or copy failed";
+    default: return "unknown status";
+  }
+}
+
+int sv_check_specs(const syn_spec* specs, int n_specs, size_t arena_bytes) {
+  return check_specs(specs, n_specs, arena_bytes);
+}
+
+int sv_check_pairs(const vc_pair* pairs, int n_pairs, size_t cand_bytes, size_t ref_bytes) {
+  return check_pairs(pairs, n_pairs, cand_bytes, ref_bytes);
+}
+
+size_t sv_generate_workspace_bytes(const syn_spec* specs, int n_specs) {
+  if (n_specs < 0 || n_specs > SV_MAX_ENTRIES || (n_specs > 0 && !specs)) return 0;
+  return spec_table_bytes(n_specs);
+}
+
+size_t sv_compare_workspace_bytes(const vc_pair* pairs, int n_pairs) {
+  if (n_pairs < 0 || n_pairs > SV_MAX_ENTRIES || (n_pairs > 0 && !pairs)) return 0;
+  for (int i = 0; i < n_pairs; ++i)
+    if (pairs[i].dtype > SV_U32) return 0;
+  return pair_table_bytes(n_pairs) + compare_partial_bytes(pairs, n_pairs);
+}
+
+size_t sv_progressive_workspace_bytes(const vc_pair* stages, int n_stages) {
+  if (n_stages < 0 || n_stages > SV_MAX_ENTRIES || (n_stages > 0 && !stages)) return 0;
+  size_t mx = 0;
+  for (int i = 0; i < n_stages; ++i) {
+    if (stages[i].dtype > SV_U32) return 0;
+    mx = std::max(mx, compare_partial_bytes(&stages[i], 1));
+  }
+  return mx;
+}
+
+int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena_bytes, void* d_ws,
+                 size_t ws_bytes, sv_stream_t stream) {
+  if (int rc = check_specs(specs, n_specs, arena_bytes)) return rc;
+  if (n_specs == 0) return SV_OK;
+  if (!d_arena) return SV_EINVAL;
+  const size_t need = spec_table_bytes(n_specs);
+  if (!ws_ok(d_ws, ws_bytes, need)) return SV_EWORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  std::vector<int> order;
+  std::vector<Group> groups;
+  group_by(n_specs, [&](int i) { return specs[i].dtype * 8u + specs[i].dist; }, order, groups);
+  std::vector<DevSpec> tab(n_specs);
+  uint64_t units = 0;
+  for (Group& g : groups) {
+    for (int k = g.begin; k < g.end; ++k) {
+      const syn_spec& s = specs[order[k]];
+      tab[k].s = s;
+      tab[k].tile_begin = g.tiles;
+      tab[k].unit_begin = units;
+      g.tiles += gen_tiles(s);
+      units += fix_units(s);
+    }
+    if (g.tiles) g.sh = generate_shape(tab[g.begin].s.dtype, tab[g.begin].s.dist, g.tiles);
+  }
+  const DevSpec* dev = nullptr;
+  if (need) {
+    if (cudaMemcpyAsync(d_ws, tab.data(), sizeof(DevSpec) * tab.size(), cudaMemcpyHostToDevice, st) != cudaSuccess)
+      return SV_ECUDA;
+    dev = static_cast<const DevSpec*>(d_ws);
+  }
+  uint8_t* arena = static_cast<uint8_t*>(d_arena);
+  cudaError_t e = cudaSuccess;
+  for (const Group& g : groups) {
+    const DevSpec& first = tab[g.begin];
+    if (first.s.dist == SV_DOTLIKE) {
+      for (int k = g.begin; e == cudaSuccess && k < g.end; ++k) e = launch_dotlike(tab[k], arena, st);
+    } else {
+      e = launch_generate_group(first.s.dtype, first.s.dist, tab.data() + g.begin, dev ? dev + g.begin : nullptr,
+                                g.end - g.begin, g.tiles, g.sh, arena, st);
+    }
+    if (e != cudaSuccess) return SV_ECUDA;
+  }
+  return status_of(launch_fixup(tab.data(), dev, n_specs, units, arena, st));
+}
+
+int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t cand_bytes, const void* d_ref,
+                   size_t ref_bytes, vc_result* d_results, void* d_ws, size_t ws_bytes, sv_stream_t stream) {
+  if (int rc = check_pairs(pairs, n_pairs, cand_bytes, ref_bytes)) return rc;
+  if (n_pairs == 0) return SV_OK;
+  if (!d_results || (cand_bytes && !d_cand) || (ref_bytes && !d_ref)) return SV_EINVAL;
+  const size_t tb = pair_table_bytes(n_pairs);
+  if (!ws_ok(d_ws, ws_bytes, tb + compare_partial_bytes(pairs, n_pairs))) return SV_EWORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  std::vector<int> order;
+  std::vector<Group> groups;
+  group_by(n_pairs, [&](int i) { return pairs[i].dtype; }, order, groups);
+  std::vector<DevPair> tab(n_pairs);
+  uint64_t slot_base = 0;
+  for (Group& g : groups) {
+    for (int k = g.begin; k < g.end; ++k) g.tiles += cmp_tiles(pairs[order[k]]);
+    g.sh = compare_shape(g.key, g.tiles);
+    uint64_t t = 0;
+    for (int k = g.begin; k < g.end; ++k) {
+      DevPair& d = tab[k];
+      d.p = pairs[order[k]];
+      d.tile_begin = t;
+      d.chunk = g.sh.chunk;
+      d.slot0 = slot_base + (uint64_t)(k - g.begin);
+      d.orig = (uint32_t)order[k];
+      d.pad = 0;
+      t += cmp_tiles(d.p);
+    }
+    slot_base += g.sh.grid + (uint64_t)(g.end - g.begin);
+  }
+  uint8_t* ws = static_cast<uint8_t*>(d_ws);
+  const DevPair* dev = nullptr;
+  if (tb) {
+    if (cudaMemcpyAsync(ws, tab.data(), sizeof(DevPair) * tab.size(), cudaMemcpyHostToDevice, st) != cudaSuccess)
+      return SV_ECUDA;
+    dev = reinterpret_cast<const DevPair*>(ws);
+  }
+  Partial* partials = reinterpret_cast<Partial*>(ws + tb);
+  const uint8_t* cand = static_cast<const uint8_t*>(d_cand);
+  const uint8_t* ref = static_cast<const uint8_t*>(d_ref);
+  for (const Group& g : groups) {
+    const cudaError_t e = launch_compare_group(g.key, tab.data() + g.begin, dev ? dev + g.begin : nullptr,
+                                               g.end - g.begin, g.tiles, g.sh, cand, ref, partials, nullptr, st);
+    if (e != cudaSuccess) return SV_ECUDA;
+  }
+  return status_of(launch_combine(tab.data(), dev, n_pairs, partials, d_results, nullptr, 0, st));
+}
+
+int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, size_t cand_bytes,
+                       const void* d_ref, size_t ref_bytes, vc_result* d_results, int32_t* d_first_failed,
+                       void* d_ws, size_t ws_bytes, sv_stream_t stream) {
+  if (int rc = check_pairs(stages, n_stages, cand_bytes, ref_bytes)) return rc;
+  if (!d_first_failed) return SV_EINVAL;
+  if (n_stages > 0 && (!d_results || (cand_bytes && !d_cand) || (ref_bytes && !d_ref))) return SV_EINVAL;
+  if (!ws_ok(d_ws, ws_bytes, sv_progressive_workspace_bytes(stages, n_stages))) return SV_EWORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(d_first_failed, 0xFF, sizeof(int32_t), st) != cudaSuccess) return SV_ECUDA;
+  Partial* partials = static_cast<Partial*>(d_ws);
+  const uint8_t* cand = static_cast<const uint8_t*>(d_cand);
+  const uint8_t* ref = static_cast<const uint8_t*>(d_ref);
+  // one compare + one combine per stage; a failed stage sets the flag and
+  // every later launch returns at its first instruction
+  for (int s = 0; s < n_stages; ++s) {
+    DevPair one;
+    one.p = stages[s];
+    one.tile_begin = 0;
+    const uint64_t tiles = cmp_tiles(stages[s]);
+    const LaunchShape sh = compare_shape(stages[s].dtype, tiles);
+    one.chunk = sh.chunk;
+    one.slot0 = 0;
+    one.orig = 0;
+    one.pad = 0;
+    cudaError_t e = launch_compare_group(stages[s].dtype, &one, nullptr, 1, tiles, sh, cand, ref, partials,
+                                         d_first_failed, st);
+    if (e == cudaSuccess) e = launch_combine(&one, nullptr, 1, partials, d_results + s, d_first_failed, s, st);
+    if (e != cudaSuccess) return SV_ECUDA;
+  }
+  return SV_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,453 @@
+// compare.cu -- verify_compare / verify_progressive kernels: functional
+// validation by Eq. 1 of CUDA-Harness (Sec. 4.2.1), per segment, sm_103a.
+//
+//   cmp_kernel      persistent; CTA b owns the contiguous tile run
+//                   [b*chunk, (b+1)*chunk) of the flat tile list (16 KiB per
+//                   operand per tile).  Four 128-bit loads per operand per
+//                   thread are issued before any arithmetic; each element is
+//                   tested with explicit fp32 round-to-nearest operations.
+//                   Statistics stay in registers until the segment ends in
+//                   this CTA's run, then warp shuffles and one shared-memory
+//                   pass give one 64-byte partial, written to slot b + segment
+//                   (unique: runs are contiguous and ordered).  No atomics.
+//   combine_kernel  one warp per segment folds its partials in CTA order
+//                   (deterministic) and writes the vc_result.
+//
+// For the progressive ladder (Sec. 4.2.2) both kernels take a device flag:
+// once a stage has failed, later stages return at once.
+//
+// Bound: HBM reads, 2 * n * sizeof(element) per segment.
+#include <float.h>
+
+#include "sv_device.cuh"
+#include "sv_kernels.h"
+
+namespace sv {
+
+struct CmpParams {
+  const DevPair* tab;  // device table, or nullptr: use inl
+  DevPair inl[SV_INLINE_ENTRIES];
+  int n;
+  uint64_t total, chunk;
+  const uint8_t* cand;
+  const uint8_t* ref;
+  Partial* partials;
+  const int32_t* flag;  // progressive: skip when *flag >= 0
+};
+
+struct CombParams {
+  const DevPair* tab;
+  DevPair inl[SV_INLINE_ENTRIES];
+  int n;
+  const Partial* partials;
+  vc_result* results;
+  int32_t* flag;
+  int stage;
+};
+
+template <class P>
+__device__ __forceinline__ const DevPair* pentry(const P& p, int i) { return p.tab ? p.tab + i : p.inl + i; }
+
+// ---------------------------------------------------------------------------
+// per-thread accumulators
+// ---------------------------------------------------------------------------
+struct Acc {
+  uint32_t mism, nan_d, inf_d, nfin;
+  uint64_t first;
+  double ssq;
+  float maxabs_f, maxrel_f;  // float types
+  uint64_t maxabs_u;         // integer types
+  double maxrel_d;           // integer types
+};
+
+__device__ __forceinline__ void acc_reset(Acc& a) {
+  a.mism = a.nan_d = a.inf_d = a.nfin = 0;
+  a.first = ~0ull;
+  a.ssq = 0.0;
+  a.maxabs_f = a.maxrel_f = 0.0f;
+  a.maxabs_u = 0;
+  a.maxrel_d = 0.0;
+}
+
+struct Tol {
+  float atol, rtol;
+  bool eqnan;
+};
+
+// one element of a float pair.  Rare outcomes (mismatch bookkeeping) are out
+// of line.  vsum / vmax collect d^2 and d over the current 16-byte vector.
+__device__ __noinline__ void float_mismatch(Acc& a, float x, float y, uint64_t idx, bool eqnan) {
+  const bool xn = x != x, yn = y != y;
+  if (xn && yn && eqnan) return;  // two NaNs match
+  a.mism++;
+  if (a.first == ~0ull) a.first = idx;
+  if (xn != yn) a.nan_d++;
+  else if (!xn && (isinf(x) || isinf(y))) a.inf_d++;
+}
+
+__device__ __forceinline__ void float_elem(Acc& a, const Tol& t, float x, float y, uint64_t idx, float& vsum,
+                                           float& vmax, float& dk) {
+  const float ay = fabsf(y);
+  const float d = fabsf(__fsub_rn(x, y));
+  const float tol = __fadd_rn(t.atol, __fmul_rn(t.rtol, ay));
+  const bool fin = (fabsf(x) <= FLT_MAX) & (ay <= FLT_MAX);
+  const bool match = (x == y) | (fin & (d <= tol));
+  if (!match) float_mismatch(a, x, y, idx, t.eqnan);
+  dk = fin ? d : 0.0f;
+  if (fin) {
+    a.nfin++;
+    vmax = fmaxf(vmax, d);
+    vsum = __fadd_rn(vsum, __fmul_rn(d, d));
+    if (ay != 0.0f) a.maxrel_f = fmaxf(a.maxrel_f, __fdiv_rn(d, ay));
+  }
+}
+
+// fold one vector's sum of squares: fp32 while it can neither overflow nor
+// lose its terms to underflow, otherwise recomputed exactly in fp64
+template <int VE>
+__device__ __forceinline__ void fold_vector(Acc& a, float vsum, float vmax, const float (&dk)[VE]) {
+  a.maxabs_f = fmaxf(a.maxabs_f, vmax);
+  if (vsum <= 0x1p120f && (vsum >= 0x1p-100f || vmax == 0.0f)) {
+    a.ssq += (double)vsum;
+  } else {
+    double s = 0.0;
+#pragma unroll
+    for (int j = 0; j < VE; ++j) s += (double)dk[j] * (double)dk[j];
+    a.ssq += s;
+  }
+}
+
+template <int DT>
+__device__ __forceinline__ void float_vector(Acc& a, const Tol& t, const uint4& xv, const uint4& yv, uint64_t idx0) {
+  constexpr int VE = 16 / elem_bytes(DT);
+  float vsum = 0.0f, vmax = 0.0f;
+  float dk[VE];
+  const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w}, ys[4] = {yv.x, yv.y, yv.z, yv.w};
+  if constexpr (DT == SV_F32) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) float_elem(a, t, __uint_as_float(xs[j]), __uint_as_float(ys[j]), idx0 + j, vsum, vmax, dk[j]);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      float_elem(a, t, to_f32<DT>(xs[j] & 0xFFFFu), to_f32<DT>(ys[j] & 0xFFFFu), idx0 + 2 * j, vsum, vmax, dk[2 * j]);
+      float_elem(a, t, to_f32<DT>(xs[j] >> 16), to_f32<DT>(ys[j] >> 16), idx0 + 2 * j + 1, vsum, vmax,
+                 dk[2 * j + 1]);
+    }
+  }
+  fold_vector<VE>(a, vsum, vmax, dk);
+}
+
+// integers: exact equality; statistics only for the (rare) unequal elements
+__device__ __noinline__ void int_mismatch(Acc& a, int64_t x, int64_t y, uint64_t idx) {
+  a.mism++;
+  if (a.first == ~0ull) a.first = idx;
+  const uint64_t d = x >= y ? (uint64_t)x - (uint64_t)y : (uint64_t)y - (uint64_t)x;
+  a.maxabs_u = d > a.maxabs_u ? d : a.maxabs_u;
+  const double dd = (double)d;
+  a.ssq += dd * dd;
+  if (y != 0) a.maxrel_d = fmax(a.maxrel_d, dd / fabs((double)y));
+}
+
+template <int DT>
+__device__ __forceinline__ void int_vector(Acc& a, const uint4& xv, const uint4& yv, uint64_t idx0) {
+  if constexpr (DT == SV_I64) {
+    const uint64_t x0 = ((uint64_t)xv.y << 32) | xv.x, x1 = ((uint64_t)xv.w << 32) | xv.z;
+    const uint64_t y0 = ((uint64_t)yv.y << 32) | yv.x, y1 = ((uint64_t)yv.w << 32) | yv.z;
+    if (x0 != y0) int_mismatch(a, (int64_t)x0, (int64_t)y0, idx0);
+    if (x1 != y1) int_mismatch(a, (int64_t)x1, (int64_t)y1, idx0 + 1);
+  } else {
+    const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w}, ys[4] = {yv.x, yv.y, yv.z, yv.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (xs[j] != ys[j]) {
+        const int64_t x = DT == SV_I32 ? (int64_t)(int32_t)xs[j] : (int64_t)xs[j];
+        const int64_t y = DT == SV_I32 ? (int64_t)(int32_t)ys[j] : (int64_t)ys[j];
+        int_mismatch(a, x, y, idx0 + j);
+      }
+    }
+  }
+}
+
+template <int DT>
+__device__ __forceinline__ void do_vector(Acc& a, const Tol& t, const uint4& xv, const uint4& yv, uint64_t idx0) {
+  if constexpr (is_float(DT)) float_vector<DT>(a, t, xv, yv, idx0);
+  else int_vector<DT>(a, xv, yv, idx0);
+}
+
+// the elements of a segment's last, partial vector, one at a time
+template <int DT>
+__device__ void do_tail(Acc& a, const Tol& t, const uint8_t* xb, const uint8_t* yb, uint64_t i0, uint64_t i1) {
+  constexpr uint32_t sz = elem_bytes(DT);
+  for (uint64_t i = i0; i < i1; ++i) {
+    if constexpr (is_float(DT)) {
+      uint32_t xr, yr;
+      if constexpr (sz == 4) {
+        xr = reinterpret_cast<const uint32_t*>(xb)[i];
+        yr = reinterpret_cast<const uint32_t*>(yb)[i];
+      } else {
+        xr = reinterpret_cast<const uint16_t*>(xb)[i];
+        yr = reinterpret_cast<const uint16_t*>(yb)[i];
+      }
+      float vsum = 0.0f, vmax = 0.0f;
+      float dk[1];
+      float_elem(a, t, to_f32<DT>(xr), to_f32<DT>(yr), i, vsum, vmax, dk[0]);
+      fold_vector<1>(a, vsum, vmax, dk);
+    } else {
+      int64_t x, y;
+      if constexpr (DT == SV_I64) {
+        x = reinterpret_cast<const int64_t*>(xb)[i];
+        y = reinterpret_cast<const int64_t*>(yb)[i];
+      } else if constexpr (DT == SV_I32) {
+        x = reinterpret_cast<const int32_t*>(xb)[i];
+        y = reinterpret_cast<const int32_t*>(yb)[i];
+      } else {
+        x = reinterpret_cast<const uint32_t*>(xb)[i];
+        y = reinterpret_cast<const uint32_t*>(yb)[i];
+      }
+      if (x != y) int_mismatch(a, x, y, i);
+    }
+  }
+}
+
+__device__ __forceinline__ uint4 ldg_stream(const uint4* p) { return __ldcs(p); }
+
+// elements [i0, i1) of one segment: i0 is tile-aligned, i1 a tile boundary or n
+template <int DT>
+__device__ void cmp_run(Acc& a, const vc_pair& pr, const uint8_t* cand, const uint8_t* ref, uint64_t i0,
+                        uint64_t i1) {
+  constexpr uint32_t sz = elem_bytes(DT), VE = 16 / sz;
+  constexpr int U = kCmpTileBytes / 16 / kThreads;  // vectors per thread per tile (4)
+  const Tol t{__double2float_rn(pr.atol), __double2float_rn(pr.rtol), (pr.flags & SV_EQUAL_NAN) != 0};
+  const uint8_t* xb = cand + pr.cand_offset;
+  const uint8_t* yb = ref + pr.ref_offset;
+  const uint4* xv = reinterpret_cast<const uint4*>(xb);
+  const uint4* yv = reinterpret_cast<const uint4*>(yb);
+  const uint64_t v0 = i0 / VE, vfull = i1 / VE;  // whole vectors in [i0, i1)
+  for (uint64_t base = v0; base < vfull; base += (uint64_t)U * kThreads) {
+    uint4 x[U], y[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint64_t v = base + (uint64_t)u * kThreads + threadIdx.x;
+      if (v < vfull) {
+        x[u] = ldg_stream(xv + v);
+        y[u] = ldg_stream(yv + v);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint64_t v = base + (uint64_t)u * kThreads + threadIdx.x;
+      if (v < vfull) do_vector<DT>(a, t, x[u], y[u], v * VE);
+    }
+  }
+  const uint64_t tail0 = vfull * VE;
+  if (tail0 < i1 && threadIdx.x == 0) do_tail<DT>(a, t, xb, yb, tail0, i1);
+}
+
+// block-wide fold of the accumulators into one partial (fixed order)
+template <bool FLOAT>
+__device__ void flush(Acc& a, Partial* out) {
+  __shared__ Partial wp[kThreads / 32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint64_t mism = a.mism, nan_d = a.nan_d, inf_d = a.inf_d, nfin = a.nfin, first = a.first;
+  double ssq = a.ssq;
+  uint64_t maxabs = FLOAT ? (uint64_t)__float_as_uint(a.maxabs_f) : a.maxabs_u;
+  double maxrel = FLOAT ? (double)a.maxrel_f : a.maxrel_d;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    mism += __shfl_down_sync(0xFFFFFFFFu, mism, o);
+    nan_d += __shfl_down_sync(0xFFFFFFFFu, nan_d, o);
+    inf_d += __shfl_down_sync(0xFFFFFFFFu, inf_d, o);
+    nfin += __shfl_down_sync(0xFFFFFFFFu, nfin, o);
+    const uint64_t f2 = __shfl_down_sync(0xFFFFFFFFu, first, o);
+    first = f2 < first ? f2 : first;
+    ssq += __shfl_down_sync(0xFFFFFFFFu, ssq, o);
+    const uint64_t m2 = __shfl_down_sync(0xFFFFFFFFu, maxabs, o);
+    maxabs = m2 > maxabs ? m2 : maxabs;  // non-negative fp32 bits order like the values
+    maxrel = fmax(maxrel, __shfl_down_sync(0xFFFFFFFFu, maxrel, o));
+  }
+  if (lane == 0) wp[w] = Partial{mism, nan_d, inf_d, nfin, first, ssq, maxabs, maxrel};
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    Partial r = wp[0];
+    for (int i = 1; i < kThreads / 32; ++i) {
+      const Partial& q = wp[i];
+      r.mism += q.mism;
+      r.nan_d += q.nan_d;
+      r.inf_d += q.inf_d;
+      r.nfin += q.nfin;
+      r.first = q.first < r.first ? q.first : r.first;
+      r.ssq += q.ssq;
+      r.maxabs = q.maxabs > r.maxabs ? q.maxabs : r.maxabs;
+      r.maxrel = fmax(r.maxrel, q.maxrel);
+    }
+    *out = r;
+  }
+  __syncthreads();
+  acc_reset(a);
+}
+
+// one instantiation per dtype; the host groups the pairs by dtype
+template <int DT>
+__global__ void __launch_bounds__(kThreads) cmp_kernel(const __grid_constant__ CmpParams p) {
+  __shared__ DevPair cur;
+  if (p.flag && *p.flag >= 0) return;  // an earlier stage failed
+  const uint64_t t0 = (uint64_t)blockIdx.x * p.chunk;
+  const uint64_t t1 = umin(t0 + p.chunk, p.total);
+  if (t0 >= t1) return;
+  int lo = 0, hi = p.n - 1;  // last segment starting at or before t0
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (pentry(p, mid)->tile_begin <= t0) lo = mid;
+    else hi = mid - 1;
+  }
+  int e = lo;
+  Acc a;
+  acc_reset(a);
+  uint64_t t = t0;
+  while (t < t1 && e < p.n) {
+    __syncthreads();
+    if (threadIdx.x == 0) cur = *pentry(p, e);
+    __syncthreads();
+    const vc_pair pr = cur.p;
+    const uint64_t tend = umin(t1, cur.tile_begin + cmp_tiles(pr));
+    if (tend > t) {
+      constexpr uint64_t te = kCmpTileBytes / elem_bytes(DT);
+      const uint64_t i0 = (t - cur.tile_begin) * te;
+      const uint64_t i1 = umin((tend - cur.tile_begin) * te, pr.n);
+      cmp_run<DT>(a, pr, p.cand, p.ref, i0, i1);
+      flush<is_float(DT)>(a, p.partials + cur.slot0 + blockIdx.x);
+      t = tend;
+    }
+    ++e;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// pass 2: one warp per segment, partials of CTAs b_first..b_last in order
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant__ CombParams p) {
+  const int e = (int)((blockIdx.x * (uint64_t)kThreads + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (e >= p.n) return;
+  const DevPair dp = *pentry(p, e);
+  vc_result* res = p.results + dp.orig;
+  if (p.flag && *p.flag >= 0) {  // skipped stage
+    if (lane == 0) {
+      vc_result r = {};
+      r.first_mismatch = -1;
+      r.state = SV_STAGE_SKIPPED;
+      *res = r;
+    }
+    return;
+  }
+  const vc_pair& pr = dp.p;
+  const bool fl = is_float(pr.dtype);
+  const uint64_t tiles = cmp_tiles(pr);
+  uint64_t mism = 0, nan_d = 0, inf_d = 0, nfin = 0, first = ~0ull, maxabs = 0;
+  double ssq = 0.0, maxrel = 0.0;
+  if (tiles) {
+    const uint64_t b0 = dp.tile_begin / dp.chunk, b1 = (dp.tile_begin + tiles - 1) / dp.chunk;
+    for (uint64_t b = b0 + lane; b <= b1; b += 32) {
+      const Partial q = p.partials[dp.slot0 + b];
+      mism += q.mism;
+      nan_d += q.nan_d;
+      inf_d += q.inf_d;
+      nfin += q.nfin;
+      first = q.first < first ? q.first : first;
+      ssq += q.ssq;
+      maxabs = q.maxabs > maxabs ? q.maxabs : maxabs;
+      maxrel = fmax(maxrel, q.maxrel);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    mism += __shfl_down_sync(0xFFFFFFFFu, mism, o);
+    nan_d += __shfl_down_sync(0xFFFFFFFFu, nan_d, o);
+    inf_d += __shfl_down_sync(0xFFFFFFFFu, inf_d, o);
+    nfin += __shfl_down_sync(0xFFFFFFFFu, nfin, o);
+    const uint64_t f2 = __shfl_down_sync(0xFFFFFFFFu, first, o);
+    first = f2 < first ? f2 : first;
+    ssq += __shfl_down_sync(0xFFFFFFFFu, ssq, o);
+    const uint64_t m2 = __shfl_down_sync(0xFFFFFFFFu, maxabs, o);
+    maxabs = m2 > maxabs ? m2 : maxabs;
+    maxrel = fmax(maxrel, __shfl_down_sync(0xFFFFFFFFu, maxrel, o));
+  }
+  if (lane != 0) return;
+  vc_result r;
+  r.mismatches = mism;
+  r.nan_disagree = nan_d;
+  r.inf_disagree = inf_d;
+  r.n_finite = fl ? nfin : pr.n;
+  r.first_mismatch = first == ~0ull ? -1 : (int64_t)first;
+  r.max_abs_u64 = fl ? 0 : maxabs;
+  r.max_abs = fl ? (double)__uint_as_float((uint32_t)maxabs) : (double)maxabs;
+  r.max_rel = maxrel;
+  r.rms = r.n_finite ? sqrt(ssq / (double)r.n_finite) : 0.0;
+  r.pass = mism == 0;
+  r.state = SV_STAGE_RUN;
+  *res = r;
+  if (p.flag && mism != 0) *p.flag = p.stage;
+}
+
+// ---------------------------------------------------------------------------
+// host launchers
+// ---------------------------------------------------------------------------
+static const void* cmp_kernel_for(uint32_t dtype) {
+  switch (dtype) {
+    case SV_F32: return reinterpret_cast<const void*>(&cmp_kernel<SV_F32>);
+    case SV_F16: return reinterpret_cast<const void*>(&cmp_kernel<SV_F16>);
+    case SV_BF16: return reinterpret_cast<const void*>(&cmp_kernel<SV_BF16>);
+    case SV_I32: return reinterpret_cast<const void*>(&cmp_kernel<SV_I32>);
+    case SV_I64: return reinterpret_cast<const void*>(&cmp_kernel<SV_I64>);
+    default: return reinterpret_cast<const void*>(&cmp_kernel<SV_U32>);
+  }
+}
+
+LaunchShape compare_shape(uint32_t dtype, uint64_t tiles) { return shape_for(tiles, grid_cap_for(cmp_kernel_for(dtype))); }
+
+template <class P>
+static void fill_pairs(P& cp, const DevPair* host, const DevPair* dev, int n) {
+  cp.tab = dev;
+  cp.n = n;
+  if (!dev)
+    for (int i = 0; i < n; ++i) cp.inl[i] = host[i];
+}
+
+cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevPair* dev, int n, uint64_t tiles,
+                                 LaunchShape sh, const uint8_t* cand, const uint8_t* ref, Partial* partials,
+                                 const int32_t* flag, cudaStream_t st) {
+  if (tiles == 0 || n == 0) return cudaSuccess;
+  CmpParams cp;
+  fill_pairs(cp, host, dev, n);
+  cp.total = tiles;
+  cp.chunk = sh.chunk;
+  cp.cand = cand;
+  cp.ref = ref;
+  cp.partials = partials;
+  cp.flag = flag;
+  switch (dtype) {
+    case SV_F32: cmp_kernel<SV_F32><<<sh.grid, kThreads, 0, st>>>(cp); break;
+    case SV_F16: cmp_kernel<SV_F16><<<sh.grid, kThreads, 0, st>>>(cp); break;
+    case SV_BF16: cmp_kernel<SV_BF16><<<sh.grid, kThreads, 0, st>>>(cp); break;
+    case SV_I32: cmp_kernel<SV_I32><<<sh.grid, kThreads, 0, st>>>(cp); break;
+    case SV_I64: cmp_kernel<SV_I64><<<sh.grid, kThreads, 0, st>>>(cp); break;
+    default: cmp_kernel<SV_U32><<<sh.grid, kThreads, 0, st>>>(cp); break;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const Partial* partials,
+                           vc_result* results, int32_t* flag, int stage, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  CombParams cp;
+  fill_pairs(cp, host, dev, n);
+  cp.partials = partials;
+  cp.results = results;
+  cp.flag = flag;
+  cp.stage = stage;
+  const uint64_t blocks = ((uint64_t)n * 32 + kThreads - 1) / kThreads;
+  combine_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(cp);
+  return cudaGetLastError();
+}
+
+}  // namespace sv

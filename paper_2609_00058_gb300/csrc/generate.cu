@@ -1,0 +1,374 @@
+// generate.cu -- syn_generate kernels: seeded synthesis of isolated test data
+// (CUDA-Harness Sec. 4.2.1), sm_103a.
+//
+//   gen_kernel    persistent, one contiguous run of 8192-element tiles per
+//                 CTA; per 4-element quantum: base values, special values,
+//                 then the clean output and (after the element-wise
+//                 perturbation) the perturbed twin, as 16-byte stores.
+//   fixup_kernel  one thread per exact-count edit (or swapped pair).
+//   dot_kernel    64 x 128 output tiles of the dot-like values with the
+//                 factors staged in shared memory; same epilogue per quantum.
+//
+// Bound: HBM writes for cheap maps; the Philox/Box-Muller ALU work for
+// normals; FP32 FMA for the dot-like values.
+#include "sv_device.cuh"
+#include "sv_kernels.h"
+
+namespace sv {
+
+struct GenParams {
+  const DevSpec* tab;  // device table, or nullptr: use inl
+  DevSpec inl[SV_INLINE_ENTRIES];
+  int n;
+  uint64_t total;  // tiles (gen) or units (fixup)
+  uint64_t chunk;  // tiles per CTA (gen)
+  uint8_t* arena;
+};
+
+__device__ __forceinline__ const DevSpec* entry(const GenParams& p, int i) { return p.tab ? p.tab + i : p.inl + i; }
+
+// last entry whose first tile/unit is <= t (entries with no tiles share their
+// successor's start, so this lands on the entry that owns t)
+template <bool UNITS>
+__device__ int find_entry(const GenParams& p, uint64_t t) {
+  int lo = 0, hi = p.n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    const uint64_t b = UNITS ? entry(p, mid)->unit_begin : entry(p, mid)->tile_begin;
+    if (b <= t) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+// stage one table entry in shared memory (all threads take part)
+__device__ __forceinline__ void stage_entry(const DevSpec* src, DevSpec* dst) {
+  static_assert(sizeof(DevSpec) % 4 == 0, "DevSpec is copied as words");
+  const uint32_t* s = reinterpret_cast<const uint32_t*>(src);
+  uint32_t* d = reinterpret_cast<uint32_t*>(dst);
+  for (int i = threadIdx.x; i < (int)(sizeof(DevSpec) / 4); i += blockDim.x) d[i] = s[i];
+}
+
+template <int DT>
+__device__ __forceinline__ void store4(uint8_t* base, uint64_t i, const typename Store<DT>::T v[4], uint32_t valid) {
+  if constexpr (elem_bytes(DT) == 4) {
+    uint32_t* p = reinterpret_cast<uint32_t*>(base) + i;
+    if (valid == 4) *reinterpret_cast<uint4*>(p) = make_uint4(v[0], v[1], v[2], v[3]);
+    else for (uint32_t j = 0; j < valid; ++j) p[j] = v[j];
+  } else if constexpr (elem_bytes(DT) == 2) {
+    uint16_t* p = reinterpret_cast<uint16_t*>(base) + i;
+    if (valid == 4) *reinterpret_cast<uint2*>(p) = make_uint2(v[0] | (v[1] << 16), v[2] | (v[3] << 16));
+    else for (uint32_t j = 0; j < valid; ++j) p[j] = (uint16_t)v[j];
+  } else {
+    uint64_t* p = reinterpret_cast<uint64_t*>(base) + i;
+    if (valid == 4) {
+      reinterpret_cast<ulonglong2*>(p)[0] = make_ulonglong2(v[0], v[1]);
+      reinterpret_cast<ulonglong2*>(p)[1] = make_ulonglong2(v[2], v[3]);
+    } else {
+      for (uint32_t j = 0; j < valid; ++j) p[j] = v[j];
+    }
+  }
+}
+
+// elements [i0, i1) of one spec, by 4-element quanta spread over the CTA
+template <int DT, int DIST>
+__device__ void gen_run(const Ctx& c, const syn_spec& s, uint64_t i0, uint64_t i1, uint8_t* arena) {
+  using T = typename Store<DT>::T;
+  uint8_t* ref = s.ref_offset == SV_NO_OUTPUT ? nullptr : arena + s.ref_offset;
+  uint8_t* cand = s.cand_offset == SV_NO_OUTPUT ? nullptr : arena + s.cand_offset;
+  const uint64_t q0 = i0 >> 2, q1 = (i1 + 3) >> 2;
+  for (uint64_t q = q0 + threadIdx.x; q < q1; q += kThreads) {
+    const uint64_t i = q << 2;
+    const uint64_t g = s.elem_offset + i;
+    const uint32_t valid = (uint32_t)umin(4, s.n - i);
+    T v[4];
+    base4<DT, DIST>(c, g, v);
+    if (c.sp_thr) specials4<DT, DIST>(c, g, v);
+    if (ref) store4<DT>(ref, i, v, valid);
+    if (cand) {
+      if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, g, v);
+      store4<DT>(cand, i, v, valid);
+    }
+  }
+}
+
+#define SV_COMBO(dt, dist) ((dt) * 8 + (dist))
+
+// one instantiation per dtype x distribution; the host groups the specs so
+// that a launch only sees its own kind
+template <int DT, int DIST>
+__global__ void __launch_bounds__(kThreads) gen_kernel(const __grid_constant__ GenParams p) {
+  __shared__ DevSpec cur;
+  const uint64_t t0 = (uint64_t)blockIdx.x * p.chunk;
+  const uint64_t t1 = umin(t0 + p.chunk, p.total);
+  if (t0 >= t1) return;
+  int e = find_entry<false>(p, t0);
+  uint64_t t = t0;
+  while (t < t1 && e < p.n) {
+    __syncthreads();  // previous entry no longer in use
+    stage_entry(entry(p, e), &cur);
+    __syncthreads();
+    const syn_spec& s = cur.s;
+    const uint64_t tend = umin(t1, cur.tile_begin + gen_tiles(s));
+    if (tend > t) {
+      const Ctx c = make_ctx(s, p.arena);
+      const uint64_t i0 = (t - cur.tile_begin) * kGenTileElems;
+      const uint64_t i1 = umin((tend - cur.tile_begin) * kGenTileElems, s.n);
+      gen_run<DT, DIST>(c, s, i0, i1, p.arena);
+      t = tend;
+    }
+    ++e;
+  }
+}
+
+// every (dtype, distribution) the streaming generator handles
+#define SV_GEN_COMBOS(X)                                                                        \
+  X(SV_F32, SV_UNIFORM) X(SV_F32, SV_NORMAL) X(SV_F32, SV_RAW_BITS) X(SV_F32, SV_CONSTANT)         \
+  X(SV_F16, SV_UNIFORM) X(SV_F16, SV_NORMAL) X(SV_F16, SV_RAW_BITS) X(SV_F16, SV_CONSTANT)         \
+  X(SV_BF16, SV_UNIFORM) X(SV_BF16, SV_NORMAL) X(SV_BF16, SV_RAW_BITS) X(SV_BF16, SV_CONSTANT)     \
+  X(SV_I32, SV_INT_RANGE) X(SV_I32, SV_PERMUTATION) X(SV_I32, SV_RAW_BITS) X(SV_I32, SV_CONSTANT)  \
+  X(SV_U32, SV_INT_RANGE) X(SV_U32, SV_PERMUTATION) X(SV_U32, SV_RAW_BITS) X(SV_U32, SV_CONSTANT)  \
+  X(SV_I64, SV_INT_RANGE) X(SV_I64, SV_PERMUTATION) X(SV_I64, SV_RAW_BITS) X(SV_I64, SV_CONSTANT)
+
+static const void* gen_kernel_for(uint32_t dtype, uint32_t dist) {
+  switch (SV_COMBO(dtype, dist)) {
+#define SV_CASE(DT, DIST) \
+  case SV_COMBO(DT, DIST): return reinterpret_cast<const void*>(&gen_kernel<DT, DIST>);
+    SV_GEN_COMBOS(SV_CASE)
+#undef SV_CASE
+    default: return nullptr;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// exact-count perturbations: one thread per selected element (per swapped
+// pair for SWAP_PAIRS); the index of stratum s of [0, N) cut into k strata is
+// floor(s N / k) + mulhi64(x, len), x from INDEX block s.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t stratum_index(const Ctx& c, uint32_t stream, uint64_t k, uint64_t st) {
+  const uint64_t start = (st * c.N) / k, end = ((st + 1) * c.N) / k;  // st < 2^21, N <= 2^40
+  const uint4 w = draw(c.key, stream, P_INDEX, st);
+  const uint64_t x = ((uint64_t)w.x << 32) | w.y;
+  return start + __umul64hi(x, end - start);
+}
+
+template <int DT, int DIST>
+__device__ void fix_one(const Ctx& c, const syn_spec& s, uint64_t u, uint8_t* arena) {
+  using T = typename Store<DT>::T;
+  const sv_perturb& pc = s.pcount;
+  uint8_t* cand = arena + s.cand_offset;
+  const uint64_t lo = s.elem_offset, hi = s.elem_offset + s.n;
+  T* out = reinterpret_cast<T*>(cand);
+  auto put = [&](uint64_t g, uint64_t v) {
+    if (g < lo || g >= hi) return;
+    const uint64_t i = g - lo;
+    if constexpr (elem_bytes(DT) == 2) reinterpret_cast<uint16_t*>(cand)[i] = (uint16_t)v;
+    else out[i] = (T)v;
+  };
+  if (pc.kind == SV_PERT_SWAP_PAIRS) {
+    const uint64_t k = 2 * pc.count;
+    const uint64_t a = stratum_index(c, pc.stream, k, 2 * u), b = stratum_index(c, pc.stream, k, 2 * u + 1);
+    const uint64_t va = value_at<DT, DIST>(c, a, 1), vb = value_at<DT, DIST>(c, b, 1);
+    put(a, vb);
+    put(b, va);
+    return;
+  }
+  const uint64_t g = stratum_index(c, pc.stream, pc.count, u);
+  if (g < lo || g >= hi) return;
+  const uint64_t v2 = value_at<DT, DIST>(c, g, 1);
+  uint64_t v3;
+  if constexpr (is_float(DT)) {
+    const float f = __double2float_rn(pc.value);
+    if (pc.kind == SV_PERT_COUNT_SET) {
+      v3 = from_f32<DT>(f);
+    } else {
+      const uint32_t b = (uint32_t)v2;
+      v3 = finite_bits<DT>(b) ? from_f32<DT>(__fadd_rn(to_f32<DT>(b), f)) : from_f32<DT>(f);
+    }
+  } else {
+    v3 = pc.kind == SV_PERT_COUNT_SET ? ((uint64_t)pc.ivalue & width_mask(DT))
+                                      : ((v2 + (uint64_t)pc.ivalue) & width_mask(DT));
+  }
+  put(g, v3);
+}
+
+__device__ void fix_dispatch(const Ctx& c, const syn_spec& s, uint64_t u, uint8_t* arena) {
+  switch (SV_COMBO(s.dtype, s.dist)) {
+#define SV_CASE(DT, DIST) \
+  case SV_COMBO(DT, DIST): fix_one<DT, DIST>(c, s, u, arena); break;
+    SV_CASE(SV_F32, SV_UNIFORM) SV_CASE(SV_F32, SV_NORMAL) SV_CASE(SV_F32, SV_RAW_BITS) SV_CASE(SV_F32, SV_CONSTANT)
+    SV_CASE(SV_F32, SV_DOTLIKE)
+    SV_CASE(SV_F16, SV_UNIFORM) SV_CASE(SV_F16, SV_NORMAL) SV_CASE(SV_F16, SV_RAW_BITS) SV_CASE(SV_F16, SV_CONSTANT)
+    SV_CASE(SV_F16, SV_DOTLIKE)
+    SV_CASE(SV_BF16, SV_UNIFORM) SV_CASE(SV_BF16, SV_NORMAL) SV_CASE(SV_BF16, SV_RAW_BITS)
+    SV_CASE(SV_BF16, SV_CONSTANT) SV_CASE(SV_BF16, SV_DOTLIKE)
+    SV_CASE(SV_I32, SV_INT_RANGE) SV_CASE(SV_I32, SV_PERMUTATION) SV_CASE(SV_I32, SV_RAW_BITS)
+    SV_CASE(SV_I32, SV_CONSTANT)
+    SV_CASE(SV_U32, SV_INT_RANGE) SV_CASE(SV_U32, SV_PERMUTATION) SV_CASE(SV_U32, SV_RAW_BITS)
+    SV_CASE(SV_U32, SV_CONSTANT)
+    SV_CASE(SV_I64, SV_INT_RANGE) SV_CASE(SV_I64, SV_PERMUTATION) SV_CASE(SV_I64, SV_RAW_BITS)
+    SV_CASE(SV_I64, SV_CONSTANT)
+#undef SV_CASE
+    default: break;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) fixup_kernel(const __grid_constant__ GenParams p) {
+  const uint64_t u = (uint64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (u >= p.total) return;
+  const DevSpec* e = entry(p, find_entry<true>(p, u));
+  const syn_spec s = e->s;
+  const Ctx c = make_ctx(s, p.arena);
+  fix_dispatch(c, s, u - e->unit_begin, p.arena);
+}
+
+// ---------------------------------------------------------------------------
+// dot-like values: 64 x 128 output tile per CTA, 8 rows x 4 columns per thread
+// (one quantum per row), factors staged in shared memory 32 k at a time; each
+// output is the k-ascending chain of fused multiply-adds.
+// ---------------------------------------------------------------------------
+constexpr int kDotRows = 64, kDotCols = 128, kDotK = 32, kDotPad = 4;
+
+struct DotParams {
+  DevSpec spec;
+  uint8_t* arena;
+  uint64_t row0;  // first row of the chunk
+};
+
+template <int DT>
+__global__ void __launch_bounds__(kThreads) dot_kernel(const __grid_constant__ DotParams p) {
+  using T = typename Store<DT>::T;
+  __shared__ __align__(16) float As[kDotK][kDotRows + kDotPad];  // A transposed: [k][row]
+  __shared__ __align__(16) float Bs[kDotK][kDotCols];
+  const syn_spec& s = p.spec.s;
+  const Ctx c = make_ctx(s, p.arena);
+  const uint64_t rows = s.rows, cols = s.cols, K = s.dot_k;
+  const uint64_t r0 = p.row0 + (uint64_t)blockIdx.y * kDotRows;
+  const uint64_t c0 = (uint64_t)blockIdx.x * kDotCols;
+  const int tid = threadIdx.x, cg = tid & 31, rg = tid >> 5;
+  float acc[8][4];
+#pragma unroll
+  for (int r = 0; r < 8; ++r)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[r][j] = 0.0f;
+
+  for (uint64_t kc = 0; kc < K; kc += kDotK) {
+    const int kn = (int)umin(kDotK, K - kc);
+    __syncthreads();
+    for (int l = tid; l < kDotRows * kDotK; l += kThreads) {  // A tile, rows x k
+      const int r = l / kDotK, k = l % kDotK;
+      const uint64_t gr = r0 + r;
+      As[k][r] = (gr < rows && k < kn) ? c.A[gr * K + kc + k] : 0.0f;
+    }
+    for (int l = tid; l < kDotK * (kDotCols / 4); l += kThreads) {  // B tile, k x cols
+      const int k = l / (kDotCols / 4), q = l % (kDotCols / 4);
+      const uint64_t gc = c0 + 4 * q;
+      float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (k < kn && gc < cols) b = *reinterpret_cast<const float4*>(c.B + (kc + k) * cols + gc);
+      *reinterpret_cast<float4*>(&Bs[k][4 * q]) = b;
+    }
+    __syncthreads();
+    for (int k = 0; k < kn; ++k) {
+      const float4 a0 = *reinterpret_cast<const float4*>(&As[k][8 * rg]);
+      const float4 a1 = *reinterpret_cast<const float4*>(&As[k][8 * rg + 4]);
+      const float4 b = *reinterpret_cast<const float4*>(&Bs[k][4 * cg]);
+      const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float bb[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+      for (int r = 0; r < 8; ++r)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[r][j] = __fmaf_rn(a[r], bb[j], acc[r][j]);
+    }
+  }
+
+  uint8_t* ref = s.ref_offset == SV_NO_OUTPUT ? nullptr : p.arena + s.ref_offset;
+  uint8_t* cand = s.cand_offset == SV_NO_OUTPUT ? nullptr : p.arena + s.cand_offset;
+  const uint64_t col = c0 + 4 * cg;
+  if (col >= cols) return;
+  const uint64_t lo = s.elem_offset, hi = s.elem_offset + s.n;
+#pragma unroll
+  for (int r = 0; r < 8; ++r) {
+    const uint64_t row = r0 + 8 * rg + r;
+    if (row >= rows) break;
+    const uint64_t g = row * cols + col;  // multiple of 4 (cols % 4 == 0)
+    if (g + 4 <= lo || g >= hi) continue;
+    T v[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) v[j] = (T)from_f32<DT>(acc[r][j]);
+    if (c.sp_thr) specials4<DT, SV_DOTLIKE>(c, g, v);
+    // chunk bounds fall on quanta (elem_offset % 4 == 0); n may end mid-quantum
+    const uint64_t i = g - lo;
+    const uint32_t valid = (uint32_t)umin(4, hi - g);
+    if (ref) store4<DT>(ref, i, v, valid);
+    if (cand) {
+      if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, g, v);
+      store4<DT>(cand, i, v, valid);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host launchers
+// ---------------------------------------------------------------------------
+static void fill_params(GenParams& gp, const DevSpec* host, const DevSpec* dev, int n) {
+  gp.tab = dev;
+  gp.n = n;
+  if (!dev)
+    for (int i = 0; i < n; ++i) gp.inl[i] = host[i];
+}
+
+LaunchShape generate_shape(uint32_t dtype, uint32_t dist, uint64_t tiles) {
+  const void* k = gen_kernel_for(dtype, dist);
+  return shape_for(tiles, k ? grid_cap_for(k) : 1);
+}
+
+cudaError_t launch_generate_group(uint32_t dtype, uint32_t dist, const DevSpec* host, const DevSpec* dev, int n,
+                                  uint64_t tiles, LaunchShape sh, uint8_t* arena, cudaStream_t st) {
+  if (tiles == 0 || n == 0) return cudaSuccess;
+  GenParams gp;
+  fill_params(gp, host, dev, n);
+  gp.total = tiles;
+  gp.chunk = sh.chunk;
+  gp.arena = arena;
+  switch (SV_COMBO(dtype, dist)) {
+#define SV_CASE(DT, DIST) \
+  case SV_COMBO(DT, DIST): gen_kernel<DT, DIST><<<sh.grid, kThreads, 0, st>>>(gp); break;
+    SV_GEN_COMBOS(SV_CASE)
+#undef SV_CASE
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_t total_units, uint8_t* arena,
+                         cudaStream_t st) {
+  if (total_units == 0) return cudaSuccess;
+  GenParams gp;
+  fill_params(gp, host, dev, n);
+  gp.total = total_units;
+  gp.chunk = 0;
+  gp.arena = arena;
+  const uint64_t blocks = (total_units + kThreads - 1) / kThreads;
+  fixup_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(gp);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dotlike(const DevSpec& spec, uint8_t* arena, cudaStream_t st) {
+  const syn_spec& s = spec.s;
+  if (s.n == 0) return cudaSuccess;
+  DotParams dp;
+  dp.spec = spec;
+  dp.arena = arena;
+  const uint64_t first_row = s.elem_offset / s.cols, last_row = (s.elem_offset + s.n - 1) / s.cols;
+  dp.row0 = first_row;
+  const dim3 grid((unsigned)((s.cols + kDotCols - 1) / kDotCols),
+                  (unsigned)((last_row - first_row + 1 + kDotRows - 1) / kDotRows));
+  switch (s.dtype) {
+    case SV_F32: dot_kernel<SV_F32><<<grid, kThreads, 0, st>>>(dp); break;
+    case SV_F16: dot_kernel<SV_F16><<<grid, kThreads, 0, st>>>(dp); break;
+    default: dot_kernel<SV_BF16><<<grid, kThreads, 0, st>>>(dp); break;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace sv

@@ -1,0 +1,93 @@
+// sv_kernels.h -- launch interface between the C-ABI layer (abi.cu) and the
+// kernels (generate.cu, compare.cu).  Internal to the library.
+//
+// Table entries are grouped by kind on the host (dtype for the compare,
+// dtype x distribution for the generator) so that every launch runs one
+// template instantiation with its own register budget and occupancy.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/synverify.h"
+
+#ifdef __CUDACC__
+#define SV_HD __host__ __device__
+#else
+#define SV_HD
+#endif
+
+namespace sv {
+
+constexpr int kThreads = 256;              // threads per CTA of every kernel
+constexpr uint32_t kGenTileElems = 8192;   // elements per generator tile
+constexpr uint32_t kCmpTileBytes = 16384;  // bytes per operand per compare tile
+constexpr uint32_t kGridCap = 4096;        // most persistent CTAs per launch
+
+// generator table entry: the caller's spec plus scheduling data
+struct DevSpec {
+  syn_spec s;
+  uint64_t tile_begin;  // first tile inside its group's tile list
+  uint64_t unit_begin;  // first thread in the exact-count fixup's list
+};
+
+// compare table entry: the caller's pair plus scheduling data
+struct DevPair {
+  vc_pair p;
+  uint64_t tile_begin;  // first tile inside its group's tile list
+  uint64_t chunk;       // tiles per CTA of its group's launch
+  uint64_t slot0;       // partial slot of CTA 0 for this pair (slot0 + b for CTA b)
+  uint32_t orig;        // index of the pair in the caller's table (result slot)
+  uint32_t pad;
+};
+
+// per-CTA partial statistics of one compare segment (64 bytes)
+struct Partial {
+  uint64_t mism, nan_d, inf_d, nfin;
+  uint64_t first;   // lowest mismatching index, UINT64_MAX if none
+  double ssq;       // sum of squared differences
+  uint64_t maxabs;  // float types: fp32 bits of max |x-y|; integers: max |x-y|
+  double maxrel;
+};
+
+struct LaunchShape {
+  uint32_t grid;   // CTAs with work
+  uint64_t chunk;  // tiles per CTA
+};
+
+// persistent grid for `tiles` tiles: at most `cap` CTAs, contiguous chunks
+LaunchShape shape_for(uint64_t tiles, uint32_t cap);
+// SMs x resident CTAs of this kernel (cached per device), at most kGridCap
+uint32_t grid_cap_for(const void* kernel);
+
+SV_HD inline uint64_t cmp_tiles(const vc_pair& p) {
+  const uint64_t sz = p.dtype == SV_I64 ? 8 : ((p.dtype == SV_F16 || p.dtype == SV_BF16) ? 2 : 4);
+  return (p.n * sz + kCmpTileBytes - 1) / kCmpTileBytes;
+}
+SV_HD inline uint64_t gen_tiles(const syn_spec& s) {
+  return s.dist == SV_DOTLIKE ? 0 : (s.n + kGenTileElems - 1) / kGenTileElems;
+}
+SV_HD inline uint64_t fix_units(const syn_spec& s) {
+  if (s.cand_offset == SV_NO_OUTPUT) return 0;
+  const uint32_t k = s.pcount.kind;
+  return (k == SV_PERT_COUNT_SET || k == SV_PERT_COUNT_ADD || k == SV_PERT_SWAP_PAIRS) ? s.pcount.count : 0;
+}
+
+// ---- generator ----
+LaunchShape generate_shape(uint32_t dtype, uint32_t dist, uint64_t tiles);
+// entries: either host (n <= SV_INLINE_ENTRIES, copied into the launch) or device
+cudaError_t launch_generate_group(uint32_t dtype, uint32_t dist, const DevSpec* host, const DevSpec* dev, int n,
+                                  uint64_t tiles, LaunchShape sh, uint8_t* arena, cudaStream_t st);
+cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_t units, uint8_t* arena,
+                         cudaStream_t st);
+cudaError_t launch_dotlike(const DevSpec& spec, uint8_t* arena, cudaStream_t st);
+
+// ---- compare ----
+LaunchShape compare_shape(uint32_t dtype, uint64_t tiles);
+cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevPair* dev, int n, uint64_t tiles,
+                                 LaunchShape sh, const uint8_t* cand, const uint8_t* ref, Partial* partials,
+                                 const int32_t* flag, cudaStream_t st);
+cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const Partial* partials,
+                           vc_result* results, int32_t* flag, int stage, cudaStream_t st);
+
+}  // namespace sv

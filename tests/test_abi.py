@@ -1,0 +1,180 @@
+"""Host-side checks of the C ABI (no GPU needed, no compute call).
+
+The library loads without a device (static CUDA runtime), exports every
+function include/synverify.h declares, its structs have the header's layout,
+and every validation error is reported before anything touches CUDA.
+"""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+import paper_2609_00058_gb300 as sv
+import workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "synverify.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_00058_gb300 import build
+    build.build()
+    return sv.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"^[A-Za-z_][\w \t\*]*?\b([a-z_][a-z0-9_]*)\s*\([^;{]*\)\s*;", text, flags=re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_the_three_entry_points():
+    names = declared_functions()
+    for n in ("syn_generate", "verify_compare", "verify_progressive"):
+        assert n in names
+
+
+def test_every_declared_function_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 10
+    for n in names:
+        assert hasattr(lib, n), n
+    assert {e[0] for e in sv.EXPORTS} == set(names)
+
+
+def test_struct_layouts():
+    assert C.sizeof(sv.syn_spec) == 224
+    assert C.sizeof(sv.vc_pair) == 48
+    assert C.sizeof(sv.vc_result) == 80
+    assert C.sizeof(sv.sv_perturb) == 40
+
+
+def test_abi_version_and_strerror(lib):
+    assert lib.sv_abi_version() == 1
+    for code in (0, -1, -2, -3, -4, -5):
+        assert lib.sv_strerror(code)
+    assert b"unknown" in lib.sv_strerror(-99)
+
+
+def _spec(**kw):
+    base = dict(dtype="f32", dist="uniform", n=1024, seed=1, ref_offset=0, p0=-1.0, p1=1.0)
+    base.update(kw)
+    return W.GenSpec(**base)
+
+
+BAD_SPECS = [
+    (dict(dtype="i32", dist="uniform"), -1),                      # float dist on an integer type
+    (dict(dtype="f32", dist="int_range"), -1),                    # integer dist on a float type
+    (dict(ref_offset=None), -1),                                   # no output at all
+    (dict(ref_offset=8), -2),                                      # misaligned output
+    (dict(elem_offset=2, logical_n=4096), -2),                     # elem_offset not a multiple of 4
+    (dict(ref_offset=4096 * 4), -3),                               # output beyond the arena
+    (dict(n=4096 * 4 + 1), -3),                                    # too many elements for the arena
+    (dict(specials=("imin",), special_rate=0.1), -1),              # integer special on a float type
+    (dict(specials=("nan",), special_rate=1.5), -1),               # rate above 1
+    (dict(specials=("nan",), special_rate=float("nan")), -1),      # NaN rate
+    (dict(p0=1.0, p1=-1.0), -1),                                   # empty uniform range
+    (dict(logical_n=100), -1),                                     # n beyond the logical length
+    (dict(logical_n=1 << 41), -3),                                 # logical length beyond the limit
+    (dict(pelem=W.Perturb("count_set", count=1)), -1),             # count kind in the element-wise slot
+    (dict(pcount=W.Perturb("rate_add_pm", rate=0.1)), -1),         # element-wise kind in the count slot
+    (dict(pcount=W.Perturb("count_set", count=0)), -1),            # empty count
+    (dict(pcount=W.Perturb("swap_pairs", count=600)), -1),         # more strata than elements
+    (dict(dtype="i32", dist="int_range", i0=5, i1=4), -1),         # empty integer range
+    (dict(dtype="i32", dist="int_range", i0=0, i1=1 << 31), -1),   # beyond int32
+    (dict(dtype="u32", dist="int_range", i0=-1, i1=3), -1),        # negative unsigned
+    (dict(dtype="i64", dist="int_range", pelem=W.Perturb("rel_noise", value=0.1)), -1),  # noise on ints
+    (dict(dtype="bf16", dist="dotlike", rows=4, cols=6, dot_k=8, n=24), -1),   # cols % 4
+    (dict(dtype="bf16", dist="dotlike", rows=4, cols=8, dot_k=8, n=24), -1),   # rows*cols != n
+    (dict(dtype="bf16", dist="dotlike", rows=4, cols=8, dot_k=8, n=32, a_offset=8), -2),
+    (dict(dtype="bf16", dist="dotlike", rows=4, cols=8, dot_k=8, n=32, b_offset=16256), -3),
+]
+
+
+@pytest.mark.parametrize("kw,code", BAD_SPECS)
+def test_invalid_specs_rejected_before_any_launch(lib, kw, code):
+    s = _spec(**kw)
+    assert sv.check_specs([s], 4096 * 4) == code
+    tab = sv.SpecTable([s])
+    # the entry point returns the same code without touching the (absent) GPU
+    assert lib.syn_generate(tab.arr, 1, 0x1000, 4096 * 4, None, 0, None) == code
+
+
+def test_valid_specs_accepted(lib):
+    ok = [_spec(), _spec(dtype="bf16", dist="normal", p0=5.0, p1=10.0, specials=("nan", "dup"), special_rate=0.1),
+          _spec(dtype="i64", dist="permutation", n=512, specials=("imin", "imax"), special_rate=0.01,
+                pcount=W.Perturb("swap_pairs", count=17)),
+          _spec(dtype="bf16", dist="dotlike", rows=4, cols=8, dot_k=8, n=32, a_offset=256, b_offset=512)]
+    for s in ok:
+        assert sv.check_specs([s], 4096 * 4) == 0
+
+
+def _pair(**kw):
+    base = dict(dtype="f32", n=1024, cand_offset=0, ref_offset=0, atol=1e-5, rtol=1e-5)
+    base.update(kw)
+    return W.Pair(**base)
+
+
+BAD_PAIRS = [
+    (dict(atol=-1.0), -1),
+    (dict(rtol=float("nan")), -1),
+    (dict(cand_offset=4), -2),
+    (dict(ref_offset=8), -2),
+    (dict(n=1025), -3),
+    (dict(dtype="i64", n=600), -3),
+    (dict(cand_offset=4096), -3),
+]
+
+
+@pytest.mark.parametrize("kw,code", BAD_PAIRS)
+def test_invalid_pairs_rejected_before_any_launch(lib, kw, code):
+    p = _pair(**kw)
+    assert sv.check_pairs([p], 4096, 4096) == code
+    tab = sv.PairTable([p])
+    assert lib.verify_compare(tab.arr, 1, 0x1000, 4096, 0x2000, 4096, 0x3000, 0x4000, 1 << 20, None) == code
+    ptab = sv.PairTable([p], progressive=True)
+    assert lib.verify_progressive(ptab.arr, 1, 0x1000, 4096, 0x2000, 4096, 0x3000, 0x5000, 0x4000, 1 << 20,
+                                  None) == code
+
+
+def test_integer_pairs_ignore_tolerances(lib):
+    assert sv.check_pairs([_pair(dtype="i32", atol=-1.0)], 4096, 4096) == 0
+
+
+def test_workspace_sizes(lib):
+    small = sv.SpecTable([_spec()] * 3)
+    assert small.ws_bytes == 0  # inline table
+    big = sv.SpecTable([_spec()] * 9)
+    assert big.ws_bytes >= 9 * 240 and big.ws_bytes % 256 == 0
+    pt = sv.PairTable([_pair()] * 3)
+    assert pt.ws_bytes >= 64 * 4 and pt.ws_bytes % 256 == 0
+    # partial slots: min(tiles, 4096) + pairs per dtype group
+    huge = sv.PairTable([_pair(n=1 << 30)])
+    assert huge.ws_bytes == ((4096 + 1) * 64 + 255) // 256 * 256
+    mixed = sv.PairTable([_pair(n=4096), _pair(dtype="bf16", n=8192), _pair(dtype="i64", n=2048)] * 4)
+    assert mixed.ws_bytes >= 12 * 80 + 24 * 64
+    lad = sv.PairTable([_pair(n=1 << e) for e in (10, 20, 27)], progressive=True)
+    assert lad.ws_bytes == ((4096 + 1) * 64 + 255) // 256 * 256
+
+
+def test_workspace_too_small_rejected(lib):
+    tab = sv.PairTable([_pair()])
+    assert lib.verify_compare(tab.arr, 1, 0x1000, 4096, 0x2000, 4096, 0x3000, 0x4000, 64, None) == -4
+    assert lib.verify_compare(tab.arr, 1, 0x1000, 4096, 0x2000, 4096, 0x3000, 0x4010, 1 << 20, None) == -4
+    big = sv.SpecTable([_spec()] * 9)
+    assert lib.syn_generate(big.arr, 9, 0x1000, 4096 * 4, None, 0, None) == -4
+
+
+def test_zero_entries_is_a_no_op(lib):
+    assert lib.syn_generate(None, 0, None, 0, None, 0, None) == 0
+    assert lib.verify_compare(None, 0, None, 0, None, 0, None, None, 0, None) == 0
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(sv, "_lib", None)
+    monkeypatch.setattr(sv, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        sv.lib()

@@ -1,0 +1,249 @@
+"""GPU parity of syn_generate (test-data synthesis, CUDA-Harness Sec. 4.2.1)
+against the CPU oracle.
+
+Bar: every stream that involves no transcendental function (uniform, integer
+range, permutation, raw bits, constants, special-value selection and kinds,
++-delta perturbations, exact-count edits, swaps, dot-like sums on the same
+factors) is bit-exact.  Box-Muller normals are computed in fp32 on the GPU:
+N(0,1) samples are within 4 ulp of the oracle's fp64-computed, fp32-rounded
+values; affine and 16-bit outputs inherit that bound (sigma * 4 ulp(z) plus
+one rounding of the output type).
+"""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2609_00058_gb300 as sv
+import workloads as W
+from gpu_util import device, ordered_16, ordered_f32, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    return device()
+
+
+def gen_both(dev, calls, size):
+    import torch
+    a = torch.zeros(size, dtype=torch.uint8, device=dev)
+    h = np.zeros(size, dtype=np.uint8)
+    for call in calls:
+        sv.generate(call, a)
+        oracle.generate(call, h)
+    torch.cuda.synchronize()
+    return a.cpu().numpy(), h
+
+
+def _view(buf, off, dtype, n):
+    t = {"f32": np.uint32, "f16": np.uint16, "bf16": np.uint16, "i32": np.uint32, "u32": np.uint32,
+         "i64": np.uint64}[dtype]
+    return buf[off: off + n * W.DTYPE_BYTES[dtype]].view(t)
+
+
+def _uses_transcendentals(spec):
+    return spec.dist == "normal" or spec.pelem.kind == "rel_noise"
+
+
+def check_spec_outputs(g, h, spec, zbound_ulp=4):
+    ref_h = _view(h, spec.ref_offset, spec.dtype, spec.n) if spec.ref_offset is not None else None
+    for role, off in ((0, spec.ref_offset), (1, spec.cand_offset)):
+        if off is None:
+            continue
+        gv, hv = _view(g, off, spec.dtype, spec.n), _view(h, off, spec.dtype, spec.n)
+        if not _uses_transcendentals(spec):
+            assert np.array_equal(gv, hv), "bit mismatch in %s/%s at %s" % (
+                spec.dtype, spec.dist, np.nonzero(gv != hv)[0][:8])
+            continue
+        if spec.dtype == "f32":
+            gf, hf = gv.view(np.float32), hv.view(np.float32)
+            fin = np.isfinite(hf)
+            assert np.array_equal(np.isfinite(gf), fin)
+            assert np.array_equal(gv[~fin], hv[~fin])  # specials are bit-exact
+            if role == 0 and spec.dist == "normal" and spec.p0 == 0.0 and spec.p1 == 1.0:
+                d = np.abs(ordered_f32(gv[fin]) - ordered_f32(hv[fin]))
+                assert d.max(initial=0) <= zbound_ulp
+                continue
+            # value bound: the clean value's z carries <= 4 ulp (scaled by
+            # sigma), every later fp32 rounding adds <= 1 ulp of its result,
+            # and the noise term c|x|z adds c|x| * 4 ulp(z) with |z| < 5.8
+            x = hf[fin].astype(np.float64)
+            xr = ref_h.view(np.float32)[fin].astype(np.float64) if ref_h is not None else x
+            sp = lambda v: np.spacing(np.abs(v).astype(np.float32)).astype(np.float64)
+            err = np.zeros_like(x)
+            if spec.dist == "normal":
+                zr = (xr - spec.p0) / spec.p1
+                err += abs(spec.p1) * zbound_ulp * sp(zr)
+            err += sp(xr) + sp(x)
+            if role == 1 and spec.pelem.kind == "rel_noise":
+                err += abs(spec.pelem.value) * np.abs(xr) * zbound_ulp * np.spacing(np.float32(5.8)) + 2 * sp(x)
+            if role == 1 and spec.pelem.kind == "rate_add_pm":
+                err += 2 * sp(x) + sp(abs(spec.pelem.value))
+            assert np.all(np.abs(gf[fin].astype(np.float64) - x) <= err * 1.0001)
+        else:
+            fin_mask = 0x7C00 if spec.dtype == "f16" else 0x7F80
+            fin = (hv & fin_mask) != fin_mask
+            assert np.array_equal((gv & fin_mask) != fin_mask, fin)
+            assert np.array_equal(gv[~fin], hv[~fin])
+            d = np.abs(ordered_16(gv[fin], spec.dtype) - ordered_16(hv[fin], spec.dtype))
+            assert d.max(initial=0) <= 1
+
+
+ALL_SPECS = [
+    dict(dtype="f32", dist="uniform", p0=-1.0, p1=1.0),
+    dict(dtype="f16", dist="uniform", p0=-100.0, p1=100.0),
+    dict(dtype="bf16", dist="uniform", p0=-100.0, p1=100.0, specials=("nan", "pinf", "denorm", "dup"),
+         special_rate=0.01),
+    dict(dtype="f32", dist="normal", p0=0.0, p1=1.0),
+    dict(dtype="f32", dist="normal", p0=5.0, p1=10.0, specials=("nan", "pinf", "ninf", "denorm", "zero", "dup"),
+         special_rate=0.05),
+    dict(dtype="bf16", dist="normal", p0=0.0, p1=1.0, specials=("nan", "denorm"), special_rate=0.02),
+    dict(dtype="f16", dist="normal", p0=0.0, p1=3.0),
+    dict(dtype="i32", dist="int_range", i0=-100, i1=100, specials=("zero", "imin", "imax", "dup"), special_rate=0.03),
+    dict(dtype="u32", dist="int_range", i0=0, i1=2**32 - 1),
+    dict(dtype="u32", dist="int_range", i0=7, i1=70000),
+    dict(dtype="i64", dist="int_range", i0=-(2**62), i1=2**62),
+    dict(dtype="i64", dist="int_range", i0=-(2**63), i1=2**63 - 1),
+    dict(dtype="i64", dist="permutation", specials=("dup", "zero", "imin", "imax"), special_rate=0.01),
+    dict(dtype="i32", dist="permutation"),
+    dict(dtype="u32", dist="permutation", logical_n=(1 << 33) // 3),
+    dict(dtype="u32", dist="raw_bits"),
+    dict(dtype="bf16", dist="raw_bits"),
+    dict(dtype="f16", dist="raw_bits"),
+    dict(dtype="i64", dist="raw_bits"),
+    dict(dtype="f32", dist="constant", p0=2.5),
+    dict(dtype="bf16", dist="constant", p0=float("nan")),
+    dict(dtype="i64", dist="constant", i0=-7),
+]
+PERTS = [
+    (W.Perturb(), W.Perturb()),
+    (W.Perturb("rate_add_pm", stream=3, rate=0.05, value=0.25, ivalue=3), W.Perturb()),
+    (W.Perturb(), W.Perturb("count_set", stream=4, count=7, value=float("nan"), ivalue=-1)),
+    (W.Perturb("rate_add_pm", stream=3, rate=0.02, value=1e-3, ivalue=1), W.Perturb("swap_pairs", stream=5, count=5)),
+    (W.Perturb(), W.Perturb("count_add", stream=6, count=3, value=1e-2, ivalue=2)),
+    (W.Perturb("rel_noise", stream=8, value=2.0 ** -9), W.Perturb("count_add", stream=6, count=2, value=1.0)),
+]
+
+
+@pytest.mark.parametrize("ki", range(len(ALL_SPECS)))
+@pytest.mark.parametrize("pi", range(len(PERTS)))
+def test_spec_matches_oracle(dev, ki, pi):
+    kw = dict(ALL_SPECS[ki])
+    pelem, pcount = PERTS[pi]
+    if kw["dtype"] not in W.FLOAT_DTYPES and pelem.kind == "rel_noise":
+        pytest.skip("rel_noise is float-only")
+    n = 3 * 8192 + 13  # several tiles and a ragged last quantum
+    sz = W.DTYPE_BYTES[kw["dtype"]]
+    ln = kw.pop("logical_n", 0)
+    spec = W.GenSpec(n=n, seed=4321, stream=9, ref_offset=0, cand_offset=(n * sz + 255) // 256 * 256,
+                     logical_n=ln, pelem=pelem, pcount=pcount, **kw)
+    g, h = gen_both(dev, [[spec]], 2 * spec.cand_offset)
+    check_spec_outputs(g, h, spec)
+
+
+def test_normal_unit_within_4_ulp_large_sample(dev):
+    n = 1 << 22
+    spec = W.GenSpec("f32", "normal", n, seed=7, stream=3, ref_offset=0, p0=0.0, p1=1.0)
+    g, h = gen_both(dev, [[spec]], 4 * n)
+    d = np.abs(ordered_f32(g.view(np.uint32)) - ordered_f32(h.view(np.uint32)))
+    assert d.max() <= 4
+    # and most are exact
+    assert (d == 0).mean() > 0.5
+
+
+def test_chunks_equal_whole_on_gpu(dev):
+    n = 50000
+    base = dict(dtype="f32", dist="uniform", seed=3, stream=1, p0=-2.0, p1=3.0, specials=("nan", "dup"),
+                special_rate=0.01, pelem=W.Perturb("rate_add_pm", stream=2, rate=0.01, value=0.5),
+                pcount=W.Perturb("swap_pairs", stream=3, count=9))
+    whole = W.GenSpec(n=n, ref_offset=0, cand_offset=4 * n, **base)
+    cuts = [0, 8192, 8196, 30000, n]
+    chunks = [W.GenSpec(n=c1 - c0, ref_offset=4 * c0, cand_offset=4 * n + 4 * c0, elem_offset=c0, logical_n=n,
+                        **base) for c0, c1 in zip(cuts[:-1], cuts[1:])]
+    import torch
+    a = torch.zeros(8 * n, dtype=torch.uint8, device=dev)
+    b = torch.zeros(8 * n, dtype=torch.uint8, device=dev)
+    sv.generate([whole], a)
+    sv.generate(chunks, b)
+    assert torch.equal(a, b)
+    h = np.zeros(8 * n, np.uint8)
+    oracle.generate([whole], h)
+    assert np.array_equal(a.cpu().numpy(), h)
+
+
+@pytest.mark.parametrize("n_specs", [1, 8, 9, 40])
+def test_many_specs_one_call(dev, n_specs):
+    # inline (<= 8) and uploaded tables, mixed kinds grouped per launch
+    kinds = [dict(dtype="f32", dist="uniform", p0=-1.0, p1=1.0),
+             dict(dtype="i32", dist="int_range", i0=-5, i1=5),
+             dict(dtype="bf16", dist="raw_bits"),
+             dict(dtype="i64", dist="permutation"),
+             dict(dtype="u32", dist="constant", i0=9)]
+    ar = W.Arena()
+    specs = []
+    for i in range(n_specs):
+        kw = kinds[i % len(kinds)]
+        n = [1, 3, 4, 5, 100, 8192, 8193, 20000][i % 8]
+        sz = W.DTYPE_BYTES[kw["dtype"]]
+        specs.append(W.GenSpec(n=n, seed=i, stream=i, ref_offset=ar.take(n * sz), cand_offset=ar.take(n * sz),
+                               specials=("zero",) if kw["dtype"] != "f32" else ("nan",), special_rate=0.1,
+                               pcount=W.Perturb("count_set", stream=1, count=1, value=7.0, ivalue=7), **kw))
+    g, h = gen_both(dev, [specs], ar.size)
+    assert np.array_equal(g, h)
+
+
+def test_dotlike_bit_exact_on_oracle_factors(dev):
+    # the factors come from the oracle; the GPU's tiled FMA chains must equal
+    # the oracle's sequential ones bit for bit
+    rows, cols, k = 200, 520, 64
+    wl = W.dotlike_bf16_pair(rows=rows, cols=cols, k=k)
+    h = np.zeros(wl.arena_bytes, np.uint8)
+    oracle.generate(wl.gen_calls[0], h)  # A and B
+    import torch
+    a = to_dev(h, dev)
+    d = wl.gen_calls[1][0]
+    sv.generate([d], a)
+    oracle.generate([d], h)
+    g = a.cpu().numpy()
+    n = rows * cols
+    assert np.array_equal(_view(g, d.ref_offset, "bf16", n), _view(h, d.ref_offset, "bf16", n))
+    gc, hc = _view(g, d.cand_offset, "bf16", n), _view(h, d.cand_offset, "bf16", n)
+    assert np.abs(ordered_16(gc, "bf16") - ordered_16(hc, "bf16")).max() <= 1
+
+
+def test_dotlike_f32_and_odd_shapes(dev):
+    for rows, cols, k in ((1, 4, 1), (65, 132, 33), (3, 256, 100)):
+        ar = W.Arena()
+        ao, bo = ar.take(4 * rows * k), ar.take(4 * k * cols)
+        ro = ar.take(4 * rows * cols)
+        fa = W.GenSpec("f32", "uniform", rows * k, seed=1, stream=0, ref_offset=ao, p0=-1, p1=1)
+        fb = W.GenSpec("f32", "uniform", k * cols, seed=1, stream=1, ref_offset=bo, p0=-1, p1=1)
+        d = W.GenSpec("f32", "dotlike", rows * cols, seed=1, stream=2, ref_offset=ro, rows=rows, cols=cols, dot_k=k,
+                      a_offset=ao, b_offset=bo, specials=("nan", "dup"), special_rate=0.01)
+        g, h = gen_both(dev, [[fa, fb], [d]], ar.size)
+        assert np.array_equal(g, h), (rows, cols, k)
+
+
+def test_dotlike_chunked(dev):
+    rows, cols, k = 40, 64, 16
+    ar = W.Arena()
+    ao, bo = ar.take(4 * rows * k), ar.take(4 * k * cols)
+    ro = ar.take(2 * rows * cols)
+    fac = [W.GenSpec("f32", "uniform", rows * k, seed=2, ref_offset=ao, p0=-1, p1=1),
+           W.GenSpec("f32", "uniform", k * cols, seed=2, stream=1, ref_offset=bo, p0=-1, p1=1)]
+    whole = W.GenSpec("bf16", "dotlike", rows * cols, seed=2, stream=2, ref_offset=ro, rows=rows, cols=cols,
+                      dot_k=k, a_offset=ao, b_offset=bo)
+    g1, h1 = gen_both(dev, [fac, [whole]], ar.size)
+    part = whole.replace(n=1000, elem_offset=704, logical_n=rows * cols, ref_offset=ro + 1408)
+    g2, _ = gen_both(dev, [fac, [part]], ar.size)
+    assert np.array_equal(g2[ro + 1408: ro + 1408 + 2000], g1[ro + 1408: ro + 1408 + 2000])
+    assert np.array_equal(g1, h1)
+
+
+def test_zero_length_and_single_element(dev):
+    specs = [W.GenSpec("f32", "uniform", 0, ref_offset=0, p0=0, p1=1),
+             W.GenSpec("i64", "permutation", 1, ref_offset=256, cand_offset=512),
+             W.GenSpec("bf16", "normal", 1, ref_offset=768, p0=0, p1=1, specials=("nan",), special_rate=1.0)]
+    g, h = gen_both(dev, [specs], 1024)
+    assert np.array_equal(g, h)

@@ -210,6 +210,14 @@ def test_permutation_is_bijection(oracle, N):
     assert np.unique(v).size == N
 
 
+def test_permutation_outside_domain_is_zero(oracle):
+    # the ragged last quantum evaluates indices >= N; with N = 5 (3-bit space),
+    # seed 3, stream 3, indices 5 and 7 are fixed points of the round map, so a
+    # walk from them would never return to [0, N): both sides return 0 there
+    assert [oracle.perm_value(5, 3, 3, g) for g in (5, 6, 7, 1 << 40)] == [0, 0, 0, 0]
+    assert sorted(oracle.perm_value(5, 3, 3, g) for g in range(5)) == list(range(5))
+
+
 def test_permutation_depends_on_seed_and_stream(oracle):
     a = oracle.perm_values(1 << 16, 5, 0, 0, 1 << 16)
     b = oracle.perm_values(1 << 16, 6, 0, 0, 1 << 16)
