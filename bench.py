@@ -1,0 +1,412 @@
+"""Benchmark of the synthesis + verification path on GB300.
+
+One step = the whole path over one batch: syn_generate of every stage's
+reference and candidate (test-data synthesis, CUDA-Harness Sec. 4.2.1) and
+verify_progressive over the stages (Eq. 1 and the fail-fast ladder,
+Sec. 4.2.2).  Default workload: the six-stage ladder n = 2^10 .. 2^27 fp32
+N(0,1) with 0.01% NaN/+-Inf/denormal injected, the candidate deviating at
+stage 4 (1.38 GB synthesized per step, 35.8 MB verified before the exit).
+
+Prints ONE JSON line (rank 0).  `value` is synthesized + verified bytes per
+second with every buffer resident in HBM; `e2e` is the same metric through
+the public API with the synthesized test data delivered to pinned host
+memory and the verdicts read back every step.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload ladder|fp32_pair|segmented|dotlike_bf16|perm_i64]
+
+Under torchrun (N > 1) every rank runs an independent replica on its own
+GPU (the path needs no exchange at this size); the time is the max over ranks.
+"""
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+METRIC = "verified GB/s and synthesized GB/s on 1 GB300, as % of HBM peak"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# dram bytes per launch of the dominant kernel from one ncu capture, keyed by
+# a hash of the kernel sources they were taken on (None once the code moves on)
+NCU_TRAFFIC = {}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+def source_hash():
+    h = hashlib.sha256()
+    d = os.path.join(ROOT, "paper_2609_00058_gb300", "csrc")
+    for f in sorted(os.listdir(d)):
+        with open(os.path.join(d, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region (NVML through ctypes; read-only)
+# ---------------------------------------------------------------------------
+REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+           0x80: "hw_power_brake_slowdown", 0x2: "applications_clocks_setting", 0x10: "sync_boost"}
+
+
+class ClockSampler:
+    def __init__(self, torch_device):
+        self.samples, self.ok, self.max_mhz = [], False, None
+        try:
+            self.nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if self.nv.nvmlInit_v2() != 0:
+                return
+            self.h = ctypes.c_void_p()
+            bus = None
+            try:
+                import torch
+                pr = torch.cuda.get_device_properties(torch_device)
+                bus = "%08x:%02x:%02x.0" % (pr.pci_domain_id, pr.pci_bus_id, pr.pci_device_id)
+            except Exception:
+                bus = None
+            rc = self.nv.nvmlDeviceGetHandleByPciBusId_v2(bus.encode(), ctypes.byref(self.h)) if bus else 1
+            if rc != 0 and self.nv.nvmlDeviceGetHandleByIndex_v2(0, ctypes.byref(self.h)) != 0:
+                return
+            m = ctypes.c_uint()
+            if self.nv.nvmlDeviceGetMaxClockInfo(self.h, 1, ctypes.byref(m)) == 0:
+                self.max_mhz = m.value
+            self.ok = True
+        except OSError:
+            pass
+
+    def _loop(self):
+        mhz, rs = ctypes.c_uint(), ctypes.c_ulonglong()
+        while not self.stop_ev.is_set():
+            if self.nv.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(mhz)) == 0 and \
+                    self.nv.nvmlDeviceGetCurrentClocksEventReasons(self.h, ctypes.byref(rs)) == 0:
+                self.samples.append((time.perf_counter(), mhz.value, rs.value))
+            time.sleep(0.002)
+
+    def start(self):
+        if not self.ok:
+            return
+        self.stop_ev = threading.Event()
+        self.th = threading.Thread(target=self._loop, daemon=True)
+        self.th.start()
+
+    def stop(self, t0, t1):
+        if not self.ok:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvml unavailable"]}
+        self.stop_ev.set()
+        self.th.join()
+        inside = [s for s in self.samples if t0 <= s[0] <= t1] or \
+            sorted(self.samples, key=lambda s: min(abs(s[0] - t0), abs(s[0] - t1)))[:3]
+        bits = 0
+        for s in inside:
+            bits |= s[2]
+        return {"sm_mhz": statistics.median(s[1] for s in inside) if inside else None,
+                "sm_max_mhz": self.max_mhz, "samples": len(inside),
+                "reasons": [v for k, v in sorted(REASONS.items()) if bits & k]}
+
+
+# ---------------------------------------------------------------------------
+# the CPU oracle on a bounded sample (baseline / reference arm)
+# ---------------------------------------------------------------------------
+def oracle_sample(workload):
+    if workload == "ladder":
+        return W.progressive_ladder((10, 14, 18, 22)), "ladder stages n=2^10,2^14,2^18,2^22 (same seeds)"
+    if workload == "fp32_pair":
+        return W.single_fp32_pair(1 << 20), "the whole fp32 pair n=2^20"
+    if workload == "segmented":
+        return W.segmented_cases(1024), "the first 1024 of the 4096 cases"
+    if workload == "dotlike_bf16":
+        return W.dotlike_bf16_pair(rows=256, cols=32768), "256 of the 32768 rows"
+    return W.int64_permutation_pair(1 << 22), "n=2^22 of the 2^28 permutation"
+
+
+def run_oracle_once(wl):
+    import oracle
+    arena = np.zeros(wl.arena_bytes, np.uint8)
+    t0 = time.perf_counter()
+    for call in wl.gen_calls:
+        oracle.generate(call, arena)
+    if wl.progressive:
+        _, ff = oracle.progressive(wl.pairs, arena, arena)
+        stages = len(wl.pairs) if ff < 0 else ff + 1
+    else:
+        oracle.compare(wl.pairs, arena, arena)
+        stages = None
+    dt = time.perf_counter() - t0
+    return dt, wl.synth_bytes() + wl.verify_bytes(stages)
+
+
+def cpu_baseline(workload):
+    wl, sample = oracle_sample(workload)
+    import oracle
+    oracle.build()
+    dt, nbytes = run_oracle_once(wl)
+    return {"value": nbytes / dt / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": sample + ", generate + verify, single-threaded C oracle, %.2f s" % dt}
+
+
+def reference_arm(args, rank, world):
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    wl, sample = oracle_sample(args.workload)
+    for _ in range(args.warmup):
+        run_oracle_once(wl)
+    times, nbytes = [], 0
+    for _ in range(args.steps):
+        dt, nbytes = run_oracle_once(wl)
+        times.append(dt)
+    tot = sum(times)
+    value = nbytes * args.steps / tot / 1e9
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded counter-based specs)",
+            "config": {"workload": wl.name, "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+def full_workload(name):
+    return W.FULL_SIZE[name]()
+
+
+def ours_arm(args, rank, world):
+    import torch
+
+    import paper_2609_00058_gb300 as sv
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    sv.lib()
+    wl = full_workload(args.workload)
+    arena = torch.zeros(wl.arena_bytes, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    spec_tabs = [sv.SpecTable(c) for c in wl.gen_calls]
+    pair_tab = sv.PairTable(wl.pairs, progressive=wl.progressive)
+    ws_bytes = max([t.ws_bytes for t in spec_tabs] + [pair_tab.ws_bytes, 256])
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    n_pairs = len(wl.pairs)
+    results = torch.empty(n_pairs * sv.RESULT_BYTES, dtype=torch.uint8, device=dev)
+    ff = torch.empty(1, dtype=torch.int32, device=dev)
+    synth_calls = [(t, c) for t, c in zip(spec_tabs, wl.gen_calls)]
+
+    def do_generate():
+        for t, _ in synth_calls:
+            sv.generate(t, arena, workspace=ws)
+
+    def do_verify():
+        if wl.progressive:
+            sv.progressive(pair_tab, arena, arena, results=results, first_failed=ff, workspace=ws)
+        else:
+            sv.compare(pair_tab, arena, arena, results=results, workspace=ws)
+
+    # one untimed pass to learn how many stages the ladder runs
+    do_generate()
+    do_verify()
+    torch.cuda.synchronize()
+    stages_run = None
+    if wl.progressive:
+        f = int(ff.item())
+        stages_run = n_pairs if f < 0 else f + 1
+    synth_b, verify_b = wl.synth_bytes(), wl.verify_bytes(stages_run)
+    step_bytes = synth_b + verify_b
+    launches_per_step = count_launches(wl)
+
+    for _ in range(args.warmup):
+        do_generate()
+        do_verify()
+    torch.cuda.synchronize()
+    barrier(world)
+
+    sampler = ClockSampler(dev)
+    sampler.start()
+    time.sleep(0.05)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    t_host0 = time.perf_counter()
+    start.record(stream)
+    for k in range(args.steps):
+        ev[k][0].record(stream)
+        do_generate()
+        ev[k][1].record(stream)
+        do_verify()
+        ev[k][2].record(stream)
+    end.record(stream)
+    torch.cuda.synchronize()
+    t_host1 = time.perf_counter()
+    barrier(world)
+    clocks = sampler.stop(t_host0, t_host1)
+    total_ms = start.elapsed_time(end)
+    gen_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / args.steps
+    ver_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / args.steps
+    total_ms = max_over_ranks(total_ms, world)
+
+    # end to end: synthesized data delivered to pinned host buffers, verdicts read back
+    host = torch.empty(wl.arena_bytes, dtype=torch.uint8, pin_memory=True)
+    host_res = torch.empty(results.numel(), dtype=torch.uint8, pin_memory=True)
+    host_ff = torch.empty(1, dtype=torch.int32, pin_memory=True)
+    out_ranges = [(s.ref_offset, s.n * W.DTYPE_BYTES[s.dtype]) for c in wl.gen_calls for s in c
+                  if s.ref_offset is not None] + \
+                 [(s.cand_offset, s.n * W.DTYPE_BYTES[s.dtype]) for c in wl.gen_calls for s in c
+                  if s.cand_offset is not None]
+    d2h = sum(n for _, n in out_ranges) + host_res.numel() + (4 if wl.progressive else 0)
+    h2d = sum(C.n * ctypes.sizeof(sv.syn_spec) for C in spec_tabs) + pair_tab.n * ctypes.sizeof(sv.vc_pair)
+
+    def e2e_step():
+        do_generate()
+        for off, nb in out_ranges:
+            host[off:off + nb].copy_(arena[off:off + nb], non_blocking=True)
+        do_verify()
+        host_res.copy_(results, non_blocking=True)
+        if wl.progressive:
+            host_ff.copy_(ff, non_blocking=True)
+        stream.synchronize()
+
+    e2e_steps = max(1, min(args.steps, 20))
+    for _ in range(min(args.warmup, 3)):
+        e2e_step()
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+
+    if rank != 0:
+        return
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    gen_bytes_launch = synth_b  # algorithmic bytes: every output element written once
+    achieved = gen_bytes_launch / (gen_ms * 1e-3) / 1e9
+    src = source_hash()
+    traffic = NCU_TRAFFIC.get((args.workload, src))
+    line = {
+        "metric": METRIC,
+        "value": world * step_bytes / (total_ms * 1e-3 / args.steps) / 1e9,
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": total_ms / args.steps,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32" if args.workload in ("ladder", "fp32_pair") else
+                 {"segmented": "mixed f32/f16/bf16/i32", "dotlike_bf16": "bf16", "perm_i64": "int64"}[args.workload],
+        "data": "synthetic (seeded counter-based specs)",
+        "config": {"workload": wl.name, "synth_bytes_per_step": synth_b, "verified_bytes_per_step": verify_b,
+                   "stages_run": stages_run, "l2": "working set %.2f GB > 129 MB L2 per step (no flush)"
+                   % (wl.arena_bytes / 1e9) if wl.arena_bytes > 2 * 129e6 else "L2 not flushed: small case",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "synth_gbs": synth_b / (gen_ms * 1e-3) / 1e9,
+        "verify_gbs": verify_b / (ver_ms * 1e-3) / 1e9,
+        "synth_frac_of_hbm": synth_b / (gen_ms * 1e-3) / 1e9 / hbm,
+        "verify_frac_of_hbm": verify_b / (ver_ms * 1e-3) / 1e9 / hbm,
+        "gen_ms": gen_ms,
+        "verify_ms": ver_ms,
+        "roofline": {"bound": "hbm", "kernel": "syn_generate (gen_kernel + exact-count fixup)",
+                     "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                     "peak_kind": "%s (%s)" % (peak_kind, "hbm_gbs"), "traffic": traffic},
+        "e2e": {"value": world * step_bytes * e2e_steps / e2e_s / 1e9, "unit": "GB/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+        "clocks": clocks,
+        "gpu_launches": launches_per_step * args.steps,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.workload)
+    print(json.dumps(line), flush=True)
+
+
+def count_launches(wl):
+    """Kernels of this library launched by one step (skipped ladder stages
+    still launch and return at once)."""
+    n = 0
+    for call in wl.gen_calls:
+        kinds = {(s.dtype, s.dist) for s in call if s.dist != "dotlike"}
+        n += len(kinds) + sum(1 for s in call if s.dist == "dotlike")
+        n += 1 if any(s.pcount.kind != "none" and s.cand_offset is not None for s in call) else 0
+    if wl.progressive:
+        n += 2 * len(wl.pairs)
+    else:
+        n += len({p.dtype for p in wl.pairs}) + 1
+    return n
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="ladder", choices=sorted(W.FULL_SIZE))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "gloo" if args.impl == "reference" else "nccl"
+        if backend == "nccl":
+            torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+        dist.init_process_group(backend)
+    if args.impl == "reference":
+        reference_arm(args, rank, world)
+    else:
+        from __graft_entry__ import build
+        if rank == 0:
+            build()
+        barrier(world)
+        build()
+        ours_arm(args, rank, world)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
