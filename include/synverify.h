@@ -233,6 +233,34 @@ int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, 
                        const void* d_ref, size_t ref_bytes, vc_result* d_results, int32_t* d_first_failed,
                        void* d_ws, size_t ws_bytes, sv_stream_t stream);
 
+/* verify_compare_noalloc: the verdicts of verify_compare for callers that
+ * cannot allocate device memory, for instance code running inside a host
+ * process whose GPU memory is owned and budgeted by another component, or on
+ * a latency-critical path that must not pay for an allocation.  Such callers
+ * pass only their inputs and outputs; the library keeps the scratch (one
+ * 64-byte partial record per CTA and pair) in a fixed array of its own device
+ * memory: SV_NOALLOC_SLOTS records, 262,656 bytes, held on every GPU that
+ * loads the library until the process exits.  The paper has no counterpart:
+ * this is a convenience of the library, not a step of the method.
+ *   Arguments and results as verify_compare, without the workspace.
+ *   Limits: at most SV_NOALLOC_MAX_PAIRS pairs, and at most SV_NOALLOC_SLOTS
+ *   partial records counted as the sum over the call's dtypes of
+ *   min(tiles, 4096) + pairs, with tiles = ceil(n * sizeof(dtype) / 16384)
+ *   summed over the pairs of that dtype (one large pair of any size fits;
+ *   two large pairs of different dtypes do not).  Beyond them: SV_ERANGE,
+ *   before anything is enqueued.
+ *   The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current) and caches it; make
+ *   that first call before any stream capture on the device.  All calls on a
+ *   device share the one array: calls whose work can overlap on the GPU race
+ *   and must be serialised by the caller.  It allocates nothing (no
+ *   cudaMalloc, no cudaFree, no allocating library routine).
+ * Errors: as verify_compare, except that SV_EWORKSPACE cannot occur. */
+#define SV_NOALLOC_MAX_PAIRS 8
+#define SV_NOALLOC_SLOTS 4104
+int verify_compare_noalloc(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t cand_bytes,
+                           const void* d_ref, size_t ref_bytes, vc_result* d_results, sv_stream_t stream);
+
 /* Static description of a status code. */
 const char* sv_strerror(int status);
 int sv_abi_version(void);

@@ -131,6 +131,7 @@ EXPORTS = [
     ("syn_generate", C.c_int, [C.POINTER(syn_spec), C.c_int, _VP, _SZ, _VP, _SZ, _VP]),
     ("verify_compare", C.c_int, [C.POINTER(vc_pair), C.c_int, _VP, _SZ, _VP, _SZ, _VP, _VP, _SZ, _VP]),
     ("verify_progressive", C.c_int, [C.POINTER(vc_pair), C.c_int, _VP, _SZ, _VP, _SZ, _VP, _VP, _VP, _SZ, _VP]),
+    ("verify_compare_noalloc", C.c_int, [C.POINTER(vc_pair), C.c_int, _VP, _SZ, _VP, _SZ, _VP, _VP]),
     ("sv_strerror", C.c_char_p, [C.c_int]),
     ("sv_abi_version", C.c_int, []),
 ]
