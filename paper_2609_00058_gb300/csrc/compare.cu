@@ -52,19 +52,20 @@ __device__ __forceinline__ const DevPair* pentry(const P& p, int i) { return p.t
 // per-thread accumulators
 // ---------------------------------------------------------------------------
 struct Acc {
-  uint32_t mism, nan_d, inf_d, nfin;
+  uint32_t mism, nan_d, inf_d, nonfin;  // nonfin: float elements outside the both-finite set
   uint64_t first;
   double ssq;
   float maxabs_f, maxrel_f;  // float types
+  float relthr;              // float types: maxrel_f * (1 - 2^-20), see float_elem
   uint64_t maxabs_u;         // integer types
   double maxrel_d;           // integer types
 };
 
 __device__ __forceinline__ void acc_reset(Acc& a) {
-  a.mism = a.nan_d = a.inf_d = a.nfin = 0;
+  a.mism = a.nan_d = a.inf_d = a.nonfin = 0;
   a.first = ~0ull;
   a.ssq = 0.0;
-  a.maxabs_f = a.maxrel_f = 0.0f;
+  a.maxabs_f = a.maxrel_f = a.relthr = 0.0f;
   a.maxabs_u = 0;
   a.maxrel_d = 0.0;
 }
@@ -74,36 +75,85 @@ struct Tol {
   bool eqnan;
 };
 
-// one element of a float pair.  Rare outcomes (mismatch bookkeeping) are out
-// of line.  vsum / vmax collect d^2 and d over the current 16-byte vector.
-__device__ __noinline__ void float_mismatch(Acc& a, float x, float y, uint64_t idx, bool eqnan) {
-  const bool xn = x != x, yn = y != y;
-  if (xn && yn && eqnan) return;  // two NaNs match
-  a.mism++;
-  if (a.first == ~0ull) a.first = idx;
-  if (xn != yn) a.nan_d++;
-  else if (!xn && (isinf(x) || isinf(y))) a.inf_d++;
-}
-
-__device__ __forceinline__ void float_elem(Acc& a, const Tol& t, float x, float y, uint64_t idx, float& vsum,
-                                           float& vmax, float& dk) {
-  const float ay = fabsf(y);
-  const float d = fabsf(__fsub_rn(x, y));
-  const float tol = __fadd_rn(t.atol, __fmul_rn(t.rtol, ay));
-  const bool fin = (fabsf(x) <= FLT_MAX) & (ay <= FLT_MAX);
-  const bool match = (x == y) | (fin & (d <= tol));
-  if (!match) float_mismatch(a, x, y, idx, t.eqnan);
-  dk = fin ? d : 0.0f;
-  if (fin) {
-    a.nfin++;
-    vmax = fmaxf(vmax, d);
-    vsum = __fadd_rn(vsum, __fmul_rn(d, d));
-    if (ay != 0.0f) a.maxrel_f = fmaxf(a.maxrel_f, __fdiv_rn(d, ay));
+// Float pairs: Eq. 1 in fp32 with explicit round-to-nearest operations.
+//
+// The hot loop handles the common case of every element: d = |x - y| <= FLT_MAX
+// (both values finite), where x == y implies d = 0 <= tol, so the verdict is
+// d <= tol alone; d and d^2 feed the per-vector max and sum.  Anything else in
+// a 16-byte vector -- a mismatch, a NaN or an infinity, a difference that
+// overflows, or an element that might raise max |x-y|/|y| -- sets one
+// predicate, and the whole vector is then re-evaluated under the full rule by
+// an out-of-line handler (float_vector_rare) that does the bookkeeping.  The
+// handler takes and returns the accumulators by value, so they never leave
+// registers on the hot path.
+//
+// max |x-y|/|y| stays exact without a division per element: fl(d/|y|) is
+// monotone in the exact quotient, so an element can raise the running maximum
+// M only if d/|y| > M, which implies d > fl(M (1 - 2^-20) |y|).
+//
+// The sum of squares (a statistic, not part of the verdict) accumulates with a
+// fused multiply-add per element, then per 16-byte vector into fp64.
+template <int DT>
+__device__ __forceinline__ void unpack_vector(const uint4& v, float (&f)[16 / elem_bytes(DT)]) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  if constexpr (DT == SV_F32) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) f[j] = __uint_as_float(w[j]);
+  } else if constexpr (DT == SV_BF16) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      f[2 * j] = __uint_as_float(w[j] << 16);
+      f[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 h = __half22float2(*reinterpret_cast<const __half2*>(&w[j]));
+      f[2 * j] = h.x;
+      f[2 * j + 1] = h.y;
+    }
   }
 }
 
-// fold one vector's sum of squares: fp32 while it can neither overflow nor
-// lose its terms to underflow, otherwise recomputed exactly in fp64
+// the full rule on one element, for the rare handler and the segment tail
+__device__ __forceinline__ void float_elem_full(Acc& a, const Tol& t, float x, float y, uint64_t idx) {
+  const float ay = fabsf(y);
+  const float d = fabsf(__fsub_rn(x, y));
+  const float tol = __fadd_rn(t.atol, __fmul_rn(t.rtol, ay));
+  const bool xn = x != x, yn = y != y;
+  const bool fin = (fabsf(x) <= FLT_MAX) & (ay <= FLT_MAX);
+  const bool match = (x == y) | (fin & (d <= tol)) | (xn & yn & t.eqnan);
+  if (!match) {
+    a.mism++;
+    if (a.first == ~0ull) a.first = idx;
+    if (xn != yn) a.nan_d++;
+    else if (!xn && (isinf(x) || ay > FLT_MAX)) a.inf_d++;
+  }
+  if (!fin) {
+    a.nonfin++;
+  } else if (!(d <= FLT_MAX)) {  // both finite, the difference overflowed
+    a.maxabs_f = d;
+    a.ssq = (double)d;
+    a.maxrel_f = d;
+    a.relthr = d;
+  } else if (ay != 0.0f && d > __fmul_rn(a.relthr, ay)) {
+    a.maxrel_f = fmaxf(a.maxrel_f, __fdiv_rn(d, ay));
+    a.relthr = __fmul_rn(a.maxrel_f, 1.0f - 0x1p-20f);
+  }
+}
+
+template <int DT>
+__device__ __noinline__ Acc float_vector_rare(Acc a, Tol t, uint4 xv, uint4 yv, uint64_t idx0) {
+  constexpr int VE = 16 / elem_bytes(DT);
+  float x[VE], y[VE];
+  unpack_vector<DT>(xv, x);
+  unpack_vector<DT>(yv, y);
+  for (int j = 0; j < VE; ++j) float_elem_full(a, t, x[j], y[j], idx0 + j);
+  return a;
+}
+
+// fold one vector's sum of squares: kept in fp32 while it can neither overflow
+// nor lose its terms to underflow, otherwise recomputed exactly in fp64
 template <int VE>
 __device__ __forceinline__ void fold_vector(Acc& a, float vsum, float vmax, const float (&dk)[VE]) {
   a.maxabs_f = fmaxf(a.maxabs_f, vmax);
@@ -120,52 +170,61 @@ __device__ __forceinline__ void fold_vector(Acc& a, float vsum, float vmax, cons
 template <int DT>
 __device__ __forceinline__ void float_vector(Acc& a, const Tol& t, const uint4& xv, const uint4& yv, uint64_t idx0) {
   constexpr int VE = 16 / elem_bytes(DT);
+  float x[VE], y[VE], dk[VE];
+  unpack_vector<DT>(xv, x);
+  unpack_vector<DT>(yv, y);
   float vsum = 0.0f, vmax = 0.0f;
-  float dk[VE];
-  const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w}, ys[4] = {yv.x, yv.y, yv.z, yv.w};
-  if constexpr (DT == SV_F32) {
+  bool rare = false;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) float_elem(a, t, __uint_as_float(xs[j]), __uint_as_float(ys[j]), idx0 + j, vsum, vmax, dk[j]);
-  } else {
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      float_elem(a, t, to_f32<DT>(xs[j] & 0xFFFFu), to_f32<DT>(ys[j] & 0xFFFFu), idx0 + 2 * j, vsum, vmax, dk[2 * j]);
-      float_elem(a, t, to_f32<DT>(xs[j] >> 16), to_f32<DT>(ys[j] >> 16), idx0 + 2 * j + 1, vsum, vmax,
-                 dk[2 * j + 1]);
-    }
+  for (int j = 0; j < VE; ++j) {
+    const float ay = fabsf(y[j]);
+    const float d = fabsf(__fsub_rn(x[j], y[j]));
+    const float tol = __fadd_rn(t.atol, __fmul_rn(t.rtol, ay));
+    const bool fin = d <= FLT_MAX;
+    rare |= !(d <= tol) | !fin | (d > __fmul_rn(a.relthr, ay));
+    dk[j] = fin ? d : 0.0f;
+    vmax = fmaxf(vmax, dk[j]);
+    vsum = __fmaf_rn(dk[j], dk[j], vsum);
   }
   fold_vector<VE>(a, vsum, vmax, dk);
+  if (rare) a = float_vector_rare<DT>(a, t, xv, yv, idx0);
 }
 
-// integers: exact equality; statistics only for the (rare) unequal elements
-__device__ __noinline__ void int_mismatch(Acc& a, int64_t x, int64_t y, uint64_t idx) {
-  a.mism++;
-  if (a.first == ~0ull) a.first = idx;
-  const uint64_t d = x >= y ? (uint64_t)x - (uint64_t)y : (uint64_t)y - (uint64_t)x;
-  a.maxabs_u = d > a.maxabs_u ? d : a.maxabs_u;
-  const double dd = (double)d;
-  a.ssq += dd * dd;
-  if (y != 0) a.maxrel_d = fmax(a.maxrel_d, dd / fabs((double)y));
+// integers: exact equality; statistics only for the (rare) unequal elements,
+// handled out of line with the accumulators passed by value
+template <int DT>
+__device__ __noinline__ Acc int_vector_rare(Acc a, uint4 xv, uint4 yv, uint64_t idx0) {
+  constexpr int VE = 16 / elem_bytes(DT);
+  int64_t x[VE], y[VE];
+  if constexpr (DT == SV_I64) {
+    x[0] = (int64_t)(((uint64_t)xv.y << 32) | xv.x);
+    x[1] = (int64_t)(((uint64_t)xv.w << 32) | xv.z);
+    y[0] = (int64_t)(((uint64_t)yv.y << 32) | yv.x);
+    y[1] = (int64_t)(((uint64_t)yv.w << 32) | yv.z);
+  } else {
+    const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w}, ys[4] = {yv.x, yv.y, yv.z, yv.w};
+    for (int j = 0; j < 4; ++j) {
+      x[j] = DT == SV_I32 ? (int64_t)(int32_t)xs[j] : (int64_t)xs[j];
+      y[j] = DT == SV_I32 ? (int64_t)(int32_t)ys[j] : (int64_t)ys[j];
+    }
+  }
+  for (int j = 0; j < VE; ++j) {
+    if (x[j] == y[j]) continue;
+    a.mism++;
+    if (a.first == ~0ull) a.first = idx0 + j;
+    const uint64_t d = x[j] >= y[j] ? (uint64_t)x[j] - (uint64_t)y[j] : (uint64_t)y[j] - (uint64_t)x[j];
+    a.maxabs_u = d > a.maxabs_u ? d : a.maxabs_u;
+    const double dd = (double)d;
+    a.ssq += dd * dd;
+    if (y[j] != 0) a.maxrel_d = fmax(a.maxrel_d, dd / fabs((double)y[j]));
+  }
+  return a;
 }
 
 template <int DT>
 __device__ __forceinline__ void int_vector(Acc& a, const uint4& xv, const uint4& yv, uint64_t idx0) {
-  if constexpr (DT == SV_I64) {
-    const uint64_t x0 = ((uint64_t)xv.y << 32) | xv.x, x1 = ((uint64_t)xv.w << 32) | xv.z;
-    const uint64_t y0 = ((uint64_t)yv.y << 32) | yv.x, y1 = ((uint64_t)yv.w << 32) | yv.z;
-    if (x0 != y0) int_mismatch(a, (int64_t)x0, (int64_t)y0, idx0);
-    if (x1 != y1) int_mismatch(a, (int64_t)x1, (int64_t)y1, idx0 + 1);
-  } else {
-    const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w}, ys[4] = {yv.x, yv.y, yv.z, yv.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (xs[j] != ys[j]) {
-        const int64_t x = DT == SV_I32 ? (int64_t)(int32_t)xs[j] : (int64_t)xs[j];
-        const int64_t y = DT == SV_I32 ? (int64_t)(int32_t)ys[j] : (int64_t)ys[j];
-        int_mismatch(a, x, y, idx0 + j);
-      }
-    }
-  }
+  const bool differ = (xv.x != yv.x) | (xv.y != yv.y) | (xv.z != yv.z) | (xv.w != yv.w);
+  if (differ) a = int_vector_rare<DT>(a, xv, yv, idx0);
 }
 
 template <int DT>
@@ -188,10 +247,13 @@ __device__ void do_tail(Acc& a, const Tol& t, const uint8_t* xb, const uint8_t* 
         xr = reinterpret_cast<const uint16_t*>(xb)[i];
         yr = reinterpret_cast<const uint16_t*>(yb)[i];
       }
-      float vsum = 0.0f, vmax = 0.0f;
-      float dk[1];
-      float_elem(a, t, to_f32<DT>(xr), to_f32<DT>(yr), i, vsum, vmax, dk[0]);
-      fold_vector<1>(a, vsum, vmax, dk);
+      const float x = to_f32<DT>(xr), y = to_f32<DT>(yr);
+      float_elem_full(a, t, x, y, i);
+      const float d = fabsf(__fsub_rn(x, y));
+      if (d <= FLT_MAX && (fabsf(x) <= FLT_MAX) && (fabsf(y) <= FLT_MAX)) {
+        a.maxabs_f = fmaxf(a.maxabs_f, d);
+        a.ssq += (double)d * (double)d;
+      }
     } else {
       int64_t x, y;
       if constexpr (DT == SV_I64) {
@@ -204,7 +266,15 @@ __device__ void do_tail(Acc& a, const Tol& t, const uint8_t* xb, const uint8_t* 
         x = reinterpret_cast<const uint32_t*>(xb)[i];
         y = reinterpret_cast<const uint32_t*>(yb)[i];
       }
-      if (x != y) int_mismatch(a, x, y, i);
+      if (x != y) {
+        a.mism++;
+        if (a.first == ~0ull) a.first = i;
+        const uint64_t d = x >= y ? (uint64_t)x - (uint64_t)y : (uint64_t)y - (uint64_t)x;
+        a.maxabs_u = d > a.maxabs_u ? d : a.maxabs_u;
+        const double dd = (double)d;
+        a.ssq += dd * dd;
+        if (y != 0) a.maxrel_d = fmax(a.maxrel_d, dd / fabs((double)y));
+      }
     }
   }
 }
@@ -233,10 +303,21 @@ __device__ void cmp_run(Acc& a, const vc_pair& pr, const uint8_t* cand, const ui
         y[u] = ldg_stream(yv + v);
       }
     }
+
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const uint64_t v = base + (uint64_t)u * kThreads + threadIdx.x;
       if (v < vfull) do_vector<DT>(a, t, x[u], y[u], v * VE);
+    }
+    if constexpr (is_float(DT)) {
+      // share the running max |x-y|/|y| across the warp: a lane only needs
+      // the exact path for an element that could raise the warp's maximum
+      // (the segment's maximum is the max over all lanes' own maxima, and an
+      // element below the warp's maximum cannot change it)
+      float m = a.maxrel_f;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+      a.relthr = __fmul_rn(m, 1.0f - 0x1p-20f);
     }
   }
   const uint64_t tail0 = vfull * VE;
@@ -248,7 +329,7 @@ template <bool FLOAT>
 __device__ void flush(Acc& a, Partial* out) {
   __shared__ Partial wp[kThreads / 32];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  uint64_t mism = a.mism, nan_d = a.nan_d, inf_d = a.inf_d, nfin = a.nfin, first = a.first;
+  uint64_t mism = a.mism, nan_d = a.nan_d, inf_d = a.inf_d, nonfin = a.nonfin, first = a.first;
   double ssq = a.ssq;
   uint64_t maxabs = FLOAT ? (uint64_t)__float_as_uint(a.maxabs_f) : a.maxabs_u;
   double maxrel = FLOAT ? (double)a.maxrel_f : a.maxrel_d;
@@ -257,7 +338,7 @@ __device__ void flush(Acc& a, Partial* out) {
     mism += __shfl_down_sync(0xFFFFFFFFu, mism, o);
     nan_d += __shfl_down_sync(0xFFFFFFFFu, nan_d, o);
     inf_d += __shfl_down_sync(0xFFFFFFFFu, inf_d, o);
-    nfin += __shfl_down_sync(0xFFFFFFFFu, nfin, o);
+    nonfin += __shfl_down_sync(0xFFFFFFFFu, nonfin, o);
     const uint64_t f2 = __shfl_down_sync(0xFFFFFFFFu, first, o);
     first = f2 < first ? f2 : first;
     ssq += __shfl_down_sync(0xFFFFFFFFu, ssq, o);
@@ -265,7 +346,7 @@ __device__ void flush(Acc& a, Partial* out) {
     maxabs = m2 > maxabs ? m2 : maxabs;  // non-negative fp32 bits order like the values
     maxrel = fmax(maxrel, __shfl_down_sync(0xFFFFFFFFu, maxrel, o));
   }
-  if (lane == 0) wp[w] = Partial{mism, nan_d, inf_d, nfin, first, ssq, maxabs, maxrel};
+  if (lane == 0) wp[w] = Partial{mism, nan_d, inf_d, nonfin, first, ssq, maxabs, maxrel};
   __syncthreads();
   if (threadIdx.x == 0) {
     Partial r = wp[0];
@@ -274,7 +355,7 @@ __device__ void flush(Acc& a, Partial* out) {
       r.mism += q.mism;
       r.nan_d += q.nan_d;
       r.inf_d += q.inf_d;
-      r.nfin += q.nfin;
+      r.nonfin += q.nonfin;
       r.first = q.first < r.first ? q.first : r.first;
       r.ssq += q.ssq;
       r.maxabs = q.maxabs > r.maxabs ? q.maxabs : r.maxabs;
@@ -288,7 +369,7 @@ __device__ void flush(Acc& a, Partial* out) {
 
 // one instantiation per dtype; the host groups the pairs by dtype
 template <int DT>
-__global__ void __launch_bounds__(kThreads) cmp_kernel(const __grid_constant__ CmpParams p) {
+__global__ void __launch_bounds__(kThreads, 3) cmp_kernel(const __grid_constant__ CmpParams p) {
   __shared__ DevPair cur;
   if (p.flag && *p.flag >= 0) return;  // an earlier stage failed
   const uint64_t t0 = (uint64_t)blockIdx.x * p.chunk;
@@ -343,7 +424,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant
   const vc_pair& pr = dp.p;
   const bool fl = is_float(pr.dtype);
   const uint64_t tiles = cmp_tiles(pr);
-  uint64_t mism = 0, nan_d = 0, inf_d = 0, nfin = 0, first = ~0ull, maxabs = 0;
+  uint64_t mism = 0, nan_d = 0, inf_d = 0, nonfin = 0, first = ~0ull, maxabs = 0;
   double ssq = 0.0, maxrel = 0.0;
   if (tiles) {
     const uint64_t b0 = dp.tile_begin / dp.chunk, b1 = (dp.tile_begin + tiles - 1) / dp.chunk;
@@ -352,7 +433,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant
       mism += q.mism;
       nan_d += q.nan_d;
       inf_d += q.inf_d;
-      nfin += q.nfin;
+      nonfin += q.nonfin;
       first = q.first < first ? q.first : first;
       ssq += q.ssq;
       maxabs = q.maxabs > maxabs ? q.maxabs : maxabs;
@@ -364,7 +445,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant
     mism += __shfl_down_sync(0xFFFFFFFFu, mism, o);
     nan_d += __shfl_down_sync(0xFFFFFFFFu, nan_d, o);
     inf_d += __shfl_down_sync(0xFFFFFFFFu, inf_d, o);
-    nfin += __shfl_down_sync(0xFFFFFFFFu, nfin, o);
+    nonfin += __shfl_down_sync(0xFFFFFFFFu, nonfin, o);
     const uint64_t f2 = __shfl_down_sync(0xFFFFFFFFu, first, o);
     first = f2 < first ? f2 : first;
     ssq += __shfl_down_sync(0xFFFFFFFFu, ssq, o);
@@ -377,7 +458,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant
   r.mismatches = mism;
   r.nan_disagree = nan_d;
   r.inf_disagree = inf_d;
-  r.n_finite = fl ? nfin : pr.n;
+  r.n_finite = fl ? pr.n - nonfin : pr.n;
   r.first_mismatch = first == ~0ull ? -1 : (int64_t)first;
   r.max_abs_u64 = fl ? 0 : maxabs;
   r.max_abs = fl ? (double)__uint_as_float((uint32_t)maxabs) : (double)maxabs;

@@ -70,24 +70,48 @@ __device__ __forceinline__ void store4(uint8_t* base, uint64_t i, const typename
   }
 }
 
-// elements [i0, i1) of one spec, by 4-element quanta spread over the CTA
-template <int DT, int DIST>
-__device__ void gen_run(const Ctx& c, const syn_spec& s, uint64_t i0, uint64_t i1, uint8_t* arena) {
+#ifndef SV_GEN_QPI
+#define SV_GEN_QPI 1  // quanta per thread per iteration (independent Philox chains)
+#endif
+#ifndef SV_GEN_MINB
+#define SV_GEN_MINB 2  // resident CTAs per SM the register budget must allow
+#endif
+
+// elements [i0, i1) of one spec, by 4-element quanta spread over the CTA.
+// `cold` is the spec's context in shared memory; the hot fields are copied to
+// registers.  Each thread carries QPI quanta at once so their Philox and
+// Box-Muller chains overlap; a quantum past the end recomputes the last one
+// and is not stored.
+template <int DT, int DIST, int QPI>
+__device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_t i1, uint8_t* arena) {
   using T = typename Store<DT>::T;
+  const Ctx c = cold;
   uint8_t* ref = s.ref_offset == SV_NO_OUTPUT ? nullptr : arena + s.ref_offset;
   uint8_t* cand = s.cand_offset == SV_NO_OUTPUT ? nullptr : arena + s.cand_offset;
+  const uint64_t eo = s.elem_offset, n = s.n;
   const uint64_t q0 = i0 >> 2, q1 = (i1 + 3) >> 2;
-  for (uint64_t q = q0 + threadIdx.x; q < q1; q += kThreads) {
-    const uint64_t i = q << 2;
-    const uint64_t g = s.elem_offset + i;
-    const uint32_t valid = (uint32_t)umin(4, s.n - i);
-    T v[4];
-    base4<DT, DIST>(c, g, v);
-    if (c.sp_thr) specials4<DT, DIST>(c, g, v);
-    if (ref) store4<DT>(ref, i, v, valid);
-    if (cand) {
-      if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, g, v);
-      store4<DT>(cand, i, v, valid);
+  for (uint64_t q = q0 + threadIdx.x; q < q1; q += (uint64_t)QPI * kThreads) {
+    T v[QPI][4];
+    uint64_t qu[QPI];
+#pragma unroll
+    for (int u = 0; u < QPI; ++u) {
+      qu[u] = umin(q + (uint64_t)u * kThreads, q1 - 1);
+      base4<DT, DIST>(c, eo + (qu[u] << 2), v[u]);
+    }
+    if (c.sp_thr) {
+#pragma unroll
+      for (int u = 0; u < QPI; ++u) specials4<DT, DIST>(c, cold, eo + (qu[u] << 2), v[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < QPI; ++u) {
+      if (q + (uint64_t)u * kThreads >= q1) break;
+      const uint64_t i = qu[u] << 2;
+      const uint32_t valid = (uint32_t)umin(4, n - i);
+      if (ref) store4<DT>(ref, i, v[u], valid);
+      if (cand) {
+        if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, cold, eo + i, v[u]);
+        store4<DT>(cand, i, v[u], valid);
+      }
     }
   }
 }
@@ -97,8 +121,9 @@ __device__ void gen_run(const Ctx& c, const syn_spec& s, uint64_t i0, uint64_t i
 // one instantiation per dtype x distribution; the host groups the specs so
 // that a launch only sees its own kind
 template <int DT, int DIST>
-__global__ void __launch_bounds__(kThreads) gen_kernel(const __grid_constant__ GenParams p) {
+__global__ void __launch_bounds__(kThreads, SV_GEN_MINB) gen_kernel(const __grid_constant__ GenParams p) {
   __shared__ DevSpec cur;
+  __shared__ Ctx ctx;
   const uint64_t t0 = (uint64_t)blockIdx.x * p.chunk;
   const uint64_t t1 = umin(t0 + p.chunk, p.total);
   if (t0 >= t1) return;
@@ -108,13 +133,14 @@ __global__ void __launch_bounds__(kThreads) gen_kernel(const __grid_constant__ G
     __syncthreads();  // previous entry no longer in use
     stage_entry(entry(p, e), &cur);
     __syncthreads();
+    if (threadIdx.x == 0) ctx = make_ctx(cur.s, p.arena);
+    __syncthreads();
     const syn_spec& s = cur.s;
     const uint64_t tend = umin(t1, cur.tile_begin + gen_tiles(s));
     if (tend > t) {
-      const Ctx c = make_ctx(s, p.arena);
       const uint64_t i0 = (t - cur.tile_begin) * kGenTileElems;
       const uint64_t i1 = umin((tend - cur.tile_begin) * kGenTileElems, s.n);
-      gen_run<DT, DIST>(c, s, i0, i1, p.arena);
+      gen_run<DT, DIST, SV_GEN_QPI>(ctx, s, i0, i1, p.arena);
       t = tend;
     }
     ++e;
@@ -147,7 +173,7 @@ static const void* gen_kernel_for(uint32_t dtype, uint32_t dist) {
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint64_t stratum_index(const Ctx& c, uint32_t stream, uint64_t k, uint64_t st) {
   const uint64_t start = (st * c.N) / k, end = ((st + 1) * c.N) / k;  // st < 2^21, N <= 2^40
-  const uint4 w = draw(c.key, stream, P_INDEX, st);
+  const uint4 w = draw(c.rk, stream, P_INDEX, st);
   const uint64_t x = ((uint64_t)w.x << 32) | w.y;
   return start + __umul64hi(x, end - start);
 }
@@ -240,8 +266,11 @@ __global__ void __launch_bounds__(kThreads) dot_kernel(const __grid_constant__ D
   using T = typename Store<DT>::T;
   __shared__ __align__(16) float As[kDotK][kDotRows + kDotPad];  // A transposed: [k][row]
   __shared__ __align__(16) float Bs[kDotK][kDotCols];
+  __shared__ Ctx cold;
   const syn_spec& s = p.spec.s;
-  const Ctx c = make_ctx(s, p.arena);
+  if (threadIdx.x == 0) cold = make_ctx(s, p.arena);
+  __syncthreads();
+  const Ctx c = cold;
   const uint64_t rows = s.rows, cols = s.cols, K = s.dot_k;
   const uint64_t r0 = p.row0 + (uint64_t)blockIdx.y * kDotRows;
   const uint64_t c0 = (uint64_t)blockIdx.x * kDotCols;
@@ -295,13 +324,13 @@ __global__ void __launch_bounds__(kThreads) dot_kernel(const __grid_constant__ D
     T v[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) v[j] = (T)from_f32<DT>(acc[r][j]);
-    if (c.sp_thr) specials4<DT, SV_DOTLIKE>(c, g, v);
+    if (c.sp_thr) specials4<DT, SV_DOTLIKE>(c, cold, g, v);
     // chunk bounds fall on quanta (elem_offset % 4 == 0); n may end mid-quantum
     const uint64_t i = g - lo;
     const uint32_t valid = (uint32_t)umin(4, hi - g);
     if (ref) store4<DT>(ref, i, v, valid);
     if (cand) {
-      if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, g, v);
+      if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, cold, g, v);
       store4<DT>(cand, i, v, valid);
     }
   }

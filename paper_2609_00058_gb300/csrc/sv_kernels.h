@@ -43,7 +43,8 @@ struct DevPair {
 
 // per-CTA partial statistics of one compare segment (64 bytes)
 struct Partial {
-  uint64_t mism, nan_d, inf_d, nfin;
+  uint64_t mism, nan_d, inf_d;
+  uint64_t nonfin;  // float types: elements with a NaN or an infinity on a side
   uint64_t first;   // lowest mismatching index, UINT64_MAX if none
   double ssq;       // sum of squared differences
   uint64_t maxabs;  // float types: fp32 bits of max |x-y|; integers: max |x-y|
