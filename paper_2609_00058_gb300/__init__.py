@@ -189,12 +189,31 @@ def to_c_pair(p) -> vc_pair:
                    p.atol, p.rtol)
 
 
+def _host_array(ctype, items):
+    """A ctypes array of `items`; tables longer than the kernel-parameter
+    capacity are placed in pinned (page-locked) host memory when a GPU is
+    present, so the library's copy of them to the device stays asynchronous."""
+    n = max(len(items), 1)
+    if len(items) > INLINE_ENTRIES:
+        try:
+            import torch
+            if torch.cuda.is_available():
+                buf = torch.empty(n * C.sizeof(ctype), dtype=torch.uint8, pin_memory=True)
+                arr = (ctype * n).from_address(buf.data_ptr())
+                for i, it in enumerate(items):
+                    arr[i] = it
+                return arr, buf
+        except (ImportError, RuntimeError):
+            pass
+    return (ctype * n)(*items), None
+
+
 class SpecTable:
     """A prepared host table of generator specs (reusable across calls)."""
 
     def __init__(self, specs: Sequence):
         self.n = len(specs)
-        self.arr = (syn_spec * max(self.n, 1))(*[to_c_spec(s) for s in specs])
+        self.arr, self._keep = _host_array(syn_spec, [to_c_spec(s) for s in specs])
         self.ws_bytes = lib().sv_generate_workspace_bytes(self.arr, self.n)
 
 
@@ -203,7 +222,7 @@ class PairTable:
 
     def __init__(self, pairs: Sequence, progressive: bool = False):
         self.n = len(pairs)
-        self.arr = (vc_pair * max(self.n, 1))(*[to_c_pair(p) for p in pairs])
+        self.arr, self._keep = _host_array(vc_pair, [to_c_pair(p) for p in pairs])
         f = lib().sv_progressive_workspace_bytes if progressive else lib().sv_compare_workspace_bytes
         self.ws_bytes = f(self.arr, self.n)
 

@@ -247,13 +247,38 @@ size_t sv_compare_workspace_bytes(const vc_pair* pairs, int n_pairs) {
   return pair_table_bytes(n_pairs) + compare_partial_bytes(pairs, n_pairs);
 }
 
+// Progressive stages run in groups: consecutive stages of one dtype, at most
+// SV_INLINE_ENTRIES of them and kStageGroupBytes of data together (a larger
+// stage is a group of its own), share one compare launch and one ordered
+// combine.  Reading a few small stages together costs less than the launches
+// it saves; the fail-fast order is applied inside the group.
+constexpr uint64_t kStageGroupBytes = 64ull << 20;
+
+static void stage_groups(const vc_pair* stages, int n, std::vector<std::pair<int, int>>& out) {
+  out.clear();
+  int b = 0;
+  while (b < n) {
+    int e = b + 1;
+    uint64_t bytes = 2 * stages[b].n * elem_bytes((int)stages[b].dtype);
+    while (e < n && e - b < SV_INLINE_ENTRIES && stages[e].dtype == stages[b].dtype) {
+      const uint64_t more = 2 * stages[e].n * elem_bytes((int)stages[e].dtype);
+      if (bytes + more > kStageGroupBytes) break;
+      bytes += more;
+      ++e;
+    }
+    out.emplace_back(b, e);
+    b = e;
+  }
+}
+
 size_t sv_progressive_workspace_bytes(const vc_pair* stages, int n_stages) {
   if (n_stages < 0 || n_stages > SV_MAX_ENTRIES || (n_stages > 0 && !stages)) return 0;
-  size_t mx = 0;
-  for (int i = 0; i < n_stages; ++i) {
+  for (int i = 0; i < n_stages; ++i)
     if (stages[i].dtype > SV_U32) return 0;
-    mx = std::max(mx, compare_partial_bytes(&stages[i], 1));
-  }
+  std::vector<std::pair<int, int>> groups;
+  stage_groups(stages, n_stages, groups);
+  size_t mx = 0;
+  for (const auto& g : groups) mx = std::max(mx, compare_partial_bytes(stages + g.first, g.second - g.first));
   return mx;
 }
 
@@ -361,21 +386,29 @@ int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, 
   Partial* partials = static_cast<Partial*>(d_ws);
   const uint8_t* cand = static_cast<const uint8_t*>(d_cand);
   const uint8_t* ref = static_cast<const uint8_t*>(d_ref);
-  // one compare + one combine per stage; a failed stage sets the flag and
-  // every later launch returns at its first instruction
-  for (int s = 0; s < n_stages; ++s) {
-    DevPair one;
-    one.p = stages[s];
-    one.tile_begin = 0;
-    const uint64_t tiles = cmp_tiles(stages[s]);
-    const LaunchShape sh = compare_shape(stages[s].dtype, tiles);
-    one.chunk = sh.chunk;
-    one.slot0 = 0;
-    one.orig = 0;
-    one.pad = 0;
-    cudaError_t e = launch_compare_group(stages[s].dtype, &one, nullptr, 1, tiles, sh, cand, ref, partials,
-                                         d_first_failed, st);
-    if (e == cudaSuccess) e = launch_combine(&one, nullptr, 1, partials, d_results + s, d_first_failed, s, st);
+  std::vector<std::pair<int, int>> groups;
+  stage_groups(stages, n_stages, groups);
+  for (const auto& g : groups) {
+    DevPair tab[SV_INLINE_ENTRIES];
+    const int ng = g.second - g.first;
+    uint64_t tiles = 0;
+    for (int k = 0; k < ng; ++k) tiles += cmp_tiles(stages[g.first + k]);
+    const uint32_t dtype = stages[g.first].dtype;
+    const LaunchShape sh = compare_shape(dtype, tiles);
+    uint64_t t = 0;
+    for (int k = 0; k < ng; ++k) {
+      tab[k].p = stages[g.first + k];
+      tab[k].tile_begin = t;
+      tab[k].chunk = sh.chunk;
+      tab[k].slot0 = (uint64_t)k;
+      tab[k].orig = (uint32_t)(g.first + k);
+      tab[k].pad = 0;
+      t += cmp_tiles(tab[k].p);
+    }
+    // the compare returns at once when an earlier group failed; the combine
+    // then reports the group as skipped
+    cudaError_t e = launch_compare_group(dtype, tab, nullptr, ng, tiles, sh, cand, ref, partials, d_first_failed, st);
+    if (e == cudaSuccess) e = launch_combine(tab, nullptr, ng, partials, d_results, d_first_failed, 0, st);
     if (e != cudaSuccess) return SV_ECUDA;
   }
   return SV_OK;

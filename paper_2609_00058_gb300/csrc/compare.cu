@@ -404,23 +404,10 @@ __global__ void __launch_bounds__(kThreads, 3) cmp_kernel(const __grid_constant_
 }
 
 // ---------------------------------------------------------------------------
-// pass 2: one warp per segment, partials of CTAs b_first..b_last in order
+// pass 2: one warp per segment folds the partials of CTAs b_first..b_last in
+// order (deterministic) into a vc_result
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant__ CombParams p) {
-  const int e = (int)((blockIdx.x * (uint64_t)kThreads + threadIdx.x) >> 5);
-  const int lane = threadIdx.x & 31;
-  if (e >= p.n) return;
-  const DevPair dp = *pentry(p, e);
-  vc_result* res = p.results + dp.orig;
-  if (p.flag && *p.flag >= 0) {  // skipped stage
-    if (lane == 0) {
-      vc_result r = {};
-      r.first_mismatch = -1;
-      r.state = SV_STAGE_SKIPPED;
-      *res = r;
-    }
-    return;
-  }
+__device__ vc_result fold_pair(const DevPair& dp, const Partial* partials, int lane) {
   const vc_pair& pr = dp.p;
   const bool fl = is_float(pr.dtype);
   const uint64_t tiles = cmp_tiles(pr);
@@ -429,7 +416,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant
   if (tiles) {
     const uint64_t b0 = dp.tile_begin / dp.chunk, b1 = (dp.tile_begin + tiles - 1) / dp.chunk;
     for (uint64_t b = b0 + lane; b <= b1; b += 32) {
-      const Partial q = p.partials[dp.slot0 + b];
+      const Partial q = partials[dp.slot0 + b];
       mism += q.mism;
       nan_d += q.nan_d;
       inf_d += q.inf_d;
@@ -453,8 +440,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant
     maxabs = m2 > maxabs ? m2 : maxabs;
     maxrel = fmax(maxrel, __shfl_down_sync(0xFFFFFFFFu, maxrel, o));
   }
-  if (lane != 0) return;
-  vc_result r;
+  vc_result r;  // meaningful in lane 0
   r.mismatches = mism;
   r.nan_disagree = nan_d;
   r.inf_disagree = inf_d;
@@ -466,8 +452,55 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant
   r.rms = r.n_finite ? sqrt(ssq / (double)r.n_finite) : 0.0;
   r.pass = mism == 0;
   r.state = SV_STAGE_RUN;
-  *res = r;
-  if (p.flag && mism != 0) *p.flag = p.stage;
+  return r;
+}
+
+__device__ __forceinline__ vc_result skipped_result() {
+  vc_result r = {};
+  r.first_mismatch = -1;
+  r.state = SV_STAGE_SKIPPED;
+  return r;
+}
+
+__global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant__ CombParams p) {
+  const int e = (int)((blockIdx.x * (uint64_t)kThreads + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (e >= p.n) return;
+  const DevPair dp = *pentry(p, e);
+  const vc_result r = fold_pair(dp, p.partials, lane);
+  if (lane == 0) p.results[dp.orig] = r;
+}
+
+// progressive ladder: one CTA folds a group of up to eight consecutive stages
+// (one warp each), then applies the fail-fast order inside the group: stages
+// after the first failing one are reported as skipped, and the flag records
+// the failing stage so that later groups do not run.  Stages of a group are
+// compared in one pass; the verdicts equal those of running them one by one.
+__global__ void __launch_bounds__(kThreads) combine_stages_kernel(const __grid_constant__ CombParams p) {
+  __shared__ vc_result res[SV_INLINE_ENTRIES];
+  const int e = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (*p.flag >= 0) {  // an earlier group failed: nothing of this group ran
+    if (threadIdx.x < p.n) p.results[pentry(p, threadIdx.x)->orig] = skipped_result();
+    return;
+  }
+  if (e < p.n) {
+    const vc_result r = fold_pair(*pentry(p, e), p.partials, lane);
+    if (lane == 0) res[e] = r;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int failed = -1;
+    for (int i = 0; i < p.n; ++i) {
+      const DevPair* dp = pentry(p, i);
+      if (failed >= 0) {
+        p.results[dp->orig] = skipped_result();
+        continue;
+      }
+      p.results[dp->orig] = res[i];
+      if (!res[i].pass) failed = (int)dp->orig;
+    }
+    if (failed >= 0) *p.flag = failed;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -526,8 +559,13 @@ cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const
   cp.results = results;
   cp.flag = flag;
   cp.stage = stage;
-  const uint64_t blocks = ((uint64_t)n * 32 + kThreads - 1) / kThreads;
-  combine_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(cp);
+  if (flag) {  // a progressive group: one CTA, stages in order
+    if (n > SV_INLINE_ENTRIES || dev) return cudaErrorInvalidValue;
+    combine_stages_kernel<<<1, kThreads, 0, st>>>(cp);
+  } else {
+    const uint64_t blocks = ((uint64_t)n * 32 + kThreads - 1) / kThreads;
+    combine_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(cp);
+  }
   return cudaGetLastError();
 }
 

@@ -286,3 +286,19 @@ def random_pair_arrays(dtype: str, n: int, seed: int, scale: float = 10.0, misma
         s2 = np.nonzero(rng.random(n) < nonfinite_frac)[0]
         arr[s2] = lim[rng.integers(0, lim.size, size=s2.size)]
     return cand.view(np.uint8), ref.view(np.uint8)
+
+
+def random_bits_pair(dtype: str, n: int, seed: int, n_changes: int) -> Tuple[np.ndarray, np.ndarray]:
+    """(cand_bytes, ref_bytes): ref = uniformly random bit patterns of the
+    dtype (every class of value: normals, denormals, zeros, infinities,
+    NaNs), cand = ref with `n_changes` random elements given new random bits
+    and as many nudged by one unit in the last place.  Cheap at any size."""
+    rng = np.random.default_rng(seed)
+    t = {2: np.uint16, 4: np.uint32, 8: np.uint64}[DTYPE_BYTES[dtype]]
+    ref = rng.integers(0, np.iinfo(t).max, size=n, dtype=t, endpoint=True)
+    cand = ref.copy()
+    idx = rng.integers(0, n, size=n_changes)
+    cand[idx] = rng.integers(0, np.iinfo(t).max, size=n_changes, dtype=t, endpoint=True)
+    idx2 = rng.integers(0, n, size=n_changes)
+    cand[idx2] = cand[idx2] + t(1)
+    return cand.view(np.uint8), ref.view(np.uint8)
