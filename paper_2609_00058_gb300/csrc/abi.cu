@@ -53,12 +53,14 @@ uint32_t grid_cap_for(const void* fn) {
   return cap;
 }
 
-LaunchShape shape_for(uint64_t tiles, uint32_t cap) {
+LaunchShape shape_for(uint64_t units, uint64_t tiles, uint32_t cap, uint64_t align) {
   LaunchShape s{0, 1};
-  if (tiles == 0) return s;
-  const uint64_t g = std::min<uint64_t>(tiles, std::max<uint32_t>(cap, 1));
-  s.chunk = (tiles + g - 1) / g;
-  s.grid = (uint32_t)((tiles + s.chunk - 1) / s.chunk);
+  if (units == 0) return s;
+  const uint64_t g = std::min<uint64_t>(std::min<uint64_t>(units, std::max<uint64_t>(tiles, 1)),
+                                        std::max<uint32_t>(cap, 1));
+  s.chunk = (units + g - 1) / g;
+  s.chunk = (s.chunk + align - 1) / align * align;  // slices start on whole loop iterations
+  s.grid = (uint32_t)((units + s.chunk - 1) / s.chunk);
   return s;
 }
 
@@ -166,7 +168,7 @@ static int check_pairs(const vc_pair* pairs, int n, size_t cb, size_t rb) {
 struct Group {
   uint32_t key;
   int begin, end;  // range in the grouped table
-  uint64_t tiles;
+  uint64_t units, tiles;
   LaunchShape sh;
 };
 
@@ -177,7 +179,7 @@ static void group_by(int n, KeyFn key, std::vector<int>& order, std::vector<Grou
   std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return key(a) < key(b); });
   groups.clear();
   for (int k = 0; k < n; ++k) {
-    if (groups.empty() || groups.back().key != key(order[k])) groups.push_back(Group{key(order[k]), k, k, 0, {0, 1}});
+    if (groups.empty() || groups.back().key != key(order[k])) groups.push_back(Group{key(order[k]), k, k, 0, 0, {0, 1}});
     groups.back().end = k + 1;
   }
 }
@@ -294,17 +296,18 @@ int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena
   std::vector<Group> groups;
   group_by(n_specs, [&](int i) { return specs[i].dtype * 8u + specs[i].dist; }, order, groups);
   std::vector<DevSpec> tab(n_specs);
-  uint64_t units = 0;
+  uint64_t fixes = 0;
   for (Group& g : groups) {
     for (int k = g.begin; k < g.end; ++k) {
       const syn_spec& s = specs[order[k]];
       tab[k].s = s;
-      tab[k].tile_begin = g.tiles;
-      tab[k].unit_begin = units;
+      tab[k].work_begin = g.units;
+      tab[k].fix_begin = fixes;
+      g.units += gen_units(s);
       g.tiles += gen_tiles(s);
-      units += fix_units(s);
+      fixes += fix_units(s);
     }
-    if (g.tiles) g.sh = generate_shape(tab[g.begin].s.dtype, tab[g.begin].s.dist, g.tiles);
+    if (g.units) g.sh = generate_shape(tab[g.begin].s.dtype, tab[g.begin].s.dist, g.units, g.tiles);
   }
   const DevSpec* dev = nullptr;
   if (need) {
@@ -320,11 +323,11 @@ int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena
       for (int k = g.begin; e == cudaSuccess && k < g.end; ++k) e = launch_dotlike(tab[k], arena, st);
     } else {
       e = launch_generate_group(first.s.dtype, first.s.dist, tab.data() + g.begin, dev ? dev + g.begin : nullptr,
-                                g.end - g.begin, g.tiles, g.sh, arena, st);
+                                g.end - g.begin, g.units, g.sh, arena, st);
     }
     if (e != cudaSuccess) return SV_ECUDA;
   }
-  return status_of(launch_fixup(tab.data(), dev, n_specs, units, arena, st));
+  return status_of(launch_fixup(tab.data(), dev, n_specs, fixes, arena, st));
 }
 
 int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t cand_bytes, const void* d_ref,
@@ -341,20 +344,23 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
   std::vector<DevPair> tab(n_pairs);
   uint64_t slot_base = 0;
   for (Group& g : groups) {
-    for (int k = g.begin; k < g.end; ++k) g.tiles += cmp_tiles(pairs[order[k]]);
-    g.sh = compare_shape(g.key, g.tiles);
-    uint64_t t = 0;
+    for (int k = g.begin; k < g.end; ++k) {
+      g.tiles += cmp_tiles(pairs[order[k]]);
+      g.units += cmp_units(pairs[order[k]]);
+    }
+    g.sh = compare_shape(g.key, g.units, g.tiles);
+    uint64_t u = 0;
     for (int k = g.begin; k < g.end; ++k) {
       DevPair& d = tab[k];
       d.p = pairs[order[k]];
-      d.tile_begin = t;
+      d.work_begin = u;
       d.chunk = g.sh.chunk;
       d.slot0 = slot_base + (uint64_t)(k - g.begin);
       d.orig = (uint32_t)order[k];
       d.pad = 0;
-      t += cmp_tiles(d.p);
+      u += cmp_units(d.p);
     }
-    slot_base += g.sh.grid + (uint64_t)(g.end - g.begin);
+    slot_base += g.sh.grid + (uint64_t)(g.end - g.begin) - 1;  // slots slot0 + b, b < grid
   }
   uint8_t* ws = static_cast<uint8_t*>(d_ws);
   const DevPair* dev = nullptr;
@@ -368,7 +374,7 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
   const uint8_t* ref = static_cast<const uint8_t*>(d_ref);
   for (const Group& g : groups) {
     const cudaError_t e = launch_compare_group(g.key, tab.data() + g.begin, dev ? dev + g.begin : nullptr,
-                                               g.end - g.begin, g.tiles, g.sh, cand, ref, partials, nullptr, st);
+                                               g.end - g.begin, g.units, g.sh, cand, ref, partials, nullptr, st);
     if (e != cudaSuccess) return SV_ECUDA;
   }
   return status_of(launch_combine(tab.data(), dev, n_pairs, partials, d_results, nullptr, 0, st));
@@ -391,23 +397,26 @@ int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, 
   for (const auto& g : groups) {
     DevPair tab[SV_INLINE_ENTRIES];
     const int ng = g.second - g.first;
-    uint64_t tiles = 0;
-    for (int k = 0; k < ng; ++k) tiles += cmp_tiles(stages[g.first + k]);
+    uint64_t tiles = 0, units = 0;
+    for (int k = 0; k < ng; ++k) {
+      tiles += cmp_tiles(stages[g.first + k]);
+      units += cmp_units(stages[g.first + k]);
+    }
     const uint32_t dtype = stages[g.first].dtype;
-    const LaunchShape sh = compare_shape(dtype, tiles);
-    uint64_t t = 0;
+    const LaunchShape sh = compare_shape(dtype, units, tiles);
+    uint64_t u = 0;
     for (int k = 0; k < ng; ++k) {
       tab[k].p = stages[g.first + k];
-      tab[k].tile_begin = t;
+      tab[k].work_begin = u;
       tab[k].chunk = sh.chunk;
       tab[k].slot0 = (uint64_t)k;
       tab[k].orig = (uint32_t)(g.first + k);
       tab[k].pad = 0;
-      t += cmp_tiles(tab[k].p);
+      u += cmp_units(tab[k].p);
     }
     // the compare returns at once when an earlier group failed; the combine
     // then reports the group as skipped
-    cudaError_t e = launch_compare_group(dtype, tab, nullptr, ng, tiles, sh, cand, ref, partials, d_first_failed, st);
+    cudaError_t e = launch_compare_group(dtype, tab, nullptr, ng, units, sh, cand, ref, partials, d_first_failed, st);
     if (e == cudaSuccess) e = launch_combine(tab, nullptr, ng, partials, d_results, d_first_failed, 0, st);
     if (e != cudaSuccess) return SV_ECUDA;
   }

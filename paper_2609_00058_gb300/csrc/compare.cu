@@ -1,9 +1,10 @@
 // compare.cu -- verify_compare / verify_progressive kernels: functional
 // validation by Eq. 1 of CUDA-Harness (Sec. 4.2.1), per segment, sm_103a.
 //
-//   cmp_kernel      persistent; CTA b owns the contiguous tile run
-//                   [b*chunk, (b+1)*chunk) of the flat tile list (16 KiB per
-//                   operand per tile).  Four 128-bit loads per operand per
+//   cmp_kernel      persistent; CTA b owns the contiguous slice
+//                   [b*chunk, (b+1)*chunk) of the weighted work units (a fixed
+//                   cost per segment plus its 16-byte vectors; 16 KiB per
+//                   operand per loop iteration).  Four 128-bit loads per operand per
 //                   thread are issued before any arithmetic; each element is
 //                   tested with explicit fp32 round-to-nearest operations.
 //                   Statistics stay in registers until the segment ends in
@@ -372,34 +373,30 @@ template <int DT>
 __global__ void __launch_bounds__(kThreads, 3) cmp_kernel(const __grid_constant__ CmpParams p) {
   __shared__ DevPair cur;
   if (p.flag && *p.flag >= 0) return;  // an earlier stage failed
-  const uint64_t t0 = (uint64_t)blockIdx.x * p.chunk;
-  const uint64_t t1 = umin(t0 + p.chunk, p.total);
-  if (t0 >= t1) return;
-  int lo = 0, hi = p.n - 1;  // last segment starting at or before t0
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (pentry(p, mid)->tile_begin <= t0) lo = mid;
-    else hi = mid - 1;
-  }
-  int e = lo;
+  __shared__ uint64_t staged[kStagedStarts];
+  const uint64_t u0 = (uint64_t)blockIdx.x * p.chunk;
+  const uint64_t u1 = umin(u0 + p.chunk, p.total);
+  if (u0 >= u1) return;
+  const int lo = find_start(pentry(p, 0), p.n, u0, staged);  // segment containing u0
   Acc a;
   acc_reset(a);
-  uint64_t t = t0;
-  while (t < t1 && e < p.n) {
+  constexpr uint64_t VE = 16 / elem_bytes(DT);
+  for (int e = lo; e < p.n; ++e) {
     __syncthreads();
     if (threadIdx.x == 0) cur = *pentry(p, e);
     __syncthreads();
+    const uint64_t wb = cur.work_begin;
+    if (wb >= u1) break;
+    const uint64_t we = wb + cmp_units(cur.p);
+    if (we <= u0) continue;
+    // this CTA overlaps the segment's units: it writes a partial for it (the
+    // combine reads one from every overlapping CTA), covering the segment's
+    // vectors that fall in [u0, u1) -- units [wb + overhead, we)
     const vc_pair pr = cur.p;
-    const uint64_t tend = umin(t1, cur.tile_begin + cmp_tiles(pr));
-    if (tend > t) {
-      constexpr uint64_t te = kCmpTileBytes / elem_bytes(DT);
-      const uint64_t i0 = (t - cur.tile_begin) * te;
-      const uint64_t i1 = umin((tend - cur.tile_begin) * te, pr.n);
-      cmp_run<DT>(a, pr, p.cand, p.ref, i0, i1);
-      flush<is_float(DT)>(a, p.partials + cur.slot0 + blockIdx.x);
-      t = tend;
-    }
-    ++e;
+    const uint64_t v_base = wb + kCmpEntryUnits;
+    const uint64_t vlo = umax(u0, v_base), vhi = umin(u1, we);
+    if (vhi > vlo) cmp_run<DT>(a, pr, p.cand, p.ref, (vlo - v_base) * VE, umin((vhi - v_base) * VE, pr.n));
+    flush<is_float(DT)>(a, p.partials + cur.slot0 + blockIdx.x);
   }
 }
 
@@ -410,11 +407,11 @@ __global__ void __launch_bounds__(kThreads, 3) cmp_kernel(const __grid_constant_
 __device__ vc_result fold_pair(const DevPair& dp, const Partial* partials, int lane) {
   const vc_pair& pr = dp.p;
   const bool fl = is_float(pr.dtype);
-  const uint64_t tiles = cmp_tiles(pr);
   uint64_t mism = 0, nan_d = 0, inf_d = 0, nonfin = 0, first = ~0ull, maxabs = 0;
   double ssq = 0.0, maxrel = 0.0;
-  if (tiles) {
-    const uint64_t b0 = dp.tile_begin / dp.chunk, b1 = (dp.tile_begin + tiles - 1) / dp.chunk;
+  {
+    // every CTA whose unit slice overlaps [work_begin, work_begin + units)
+    const uint64_t b0 = dp.work_begin / dp.chunk, b1 = (dp.work_begin + cmp_units(pr) - 1) / dp.chunk;
     for (uint64_t b = b0 + lane; b <= b1; b += 32) {
       const Partial q = partials[dp.slot0 + b];
       mism += q.mism;
@@ -517,7 +514,9 @@ static const void* cmp_kernel_for(uint32_t dtype) {
   }
 }
 
-LaunchShape compare_shape(uint32_t dtype, uint64_t tiles) { return shape_for(tiles, grid_cap_for(cmp_kernel_for(dtype))); }
+LaunchShape compare_shape(uint32_t dtype, uint64_t units, uint64_t tiles) {
+  return shape_for(units, tiles, grid_cap_for(cmp_kernel_for(dtype)), kCmpTileBytes / 16);
+}
 
 template <class P>
 static void fill_pairs(P& cp, const DevPair* host, const DevPair* dev, int n) {
@@ -527,13 +526,13 @@ static void fill_pairs(P& cp, const DevPair* host, const DevPair* dev, int n) {
     for (int i = 0; i < n; ++i) cp.inl[i] = host[i];
 }
 
-cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevPair* dev, int n, uint64_t tiles,
+cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevPair* dev, int n, uint64_t units,
                                  LaunchShape sh, const uint8_t* cand, const uint8_t* ref, Partial* partials,
                                  const int32_t* flag, cudaStream_t st) {
-  if (tiles == 0 || n == 0) return cudaSuccess;
+  if (units == 0 || n == 0) return cudaSuccess;
   CmpParams cp;
   fill_pairs(cp, host, dev, n);
-  cp.total = tiles;
+  cp.total = units;
   cp.chunk = sh.chunk;
   cp.cand = cand;
   cp.ref = ref;

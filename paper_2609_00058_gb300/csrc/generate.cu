@@ -1,7 +1,7 @@
 // generate.cu -- syn_generate kernels: seeded synthesis of isolated test data
 // (CUDA-Harness Sec. 4.2.1), sm_103a.
 //
-//   gen_kernel    persistent, one contiguous run of 8192-element tiles per
+//   gen_kernel    persistent, one contiguous slice of weighted work units per
 //                 CTA; per 4-element quantum: base values, special values,
 //                 then the clean output and (after the element-wise
 //                 perturbation) the perturbed twin, as 16-byte stores.
@@ -20,21 +20,20 @@ struct GenParams {
   const DevSpec* tab;  // device table, or nullptr: use inl
   DevSpec inl[SV_INLINE_ENTRIES];
   int n;
-  uint64_t total;  // tiles (gen) or units (fixup)
-  uint64_t chunk;  // tiles per CTA (gen)
+  uint64_t total;  // weighted units (gen) or edits (fixup)
+  uint64_t chunk;  // units per CTA (gen)
   uint8_t* arena;
 };
 
 __device__ __forceinline__ const DevSpec* entry(const GenParams& p, int i) { return p.tab ? p.tab + i : p.inl + i; }
 
-// last entry whose first tile/unit is <= t (entries with no tiles share their
-// successor's start, so this lands on the entry that owns t)
-template <bool UNITS>
-__device__ int find_entry(const GenParams& p, uint64_t t) {
+// last entry whose first fixup edit is <= t (entries with no edits share their
+// successor's start, so this lands on the entry owning t)
+__device__ int find_fix_entry(const GenParams& p, uint64_t t) {
   int lo = 0, hi = p.n - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    const uint64_t b = UNITS ? entry(p, mid)->unit_begin : entry(p, mid)->tile_begin;
+    const uint64_t b = entry(p, mid)->fix_begin;
     if (b <= t) lo = mid;
     else hi = mid - 1;
   }
@@ -124,26 +123,24 @@ template <int DT, int DIST>
 __global__ void __launch_bounds__(kThreads, SV_GEN_MINB) gen_kernel(const __grid_constant__ GenParams p) {
   __shared__ DevSpec cur;
   __shared__ Ctx ctx;
-  const uint64_t t0 = (uint64_t)blockIdx.x * p.chunk;
-  const uint64_t t1 = umin(t0 + p.chunk, p.total);
-  if (t0 >= t1) return;
-  int e = find_entry<false>(p, t0);
-  uint64_t t = t0;
-  while (t < t1 && e < p.n) {
+  __shared__ uint64_t staged[kStagedStarts];
+  const uint64_t u0 = (uint64_t)blockIdx.x * p.chunk;
+  const uint64_t u1 = umin(u0 + p.chunk, p.total);
+  if (u0 >= u1) return;
+  for (int e = find_start(entry(p, 0), p.n, u0, staged); e < p.n; ++e) {
     __syncthreads();  // previous entry no longer in use
     stage_entry(entry(p, e), &cur);
     __syncthreads();
+    const uint64_t wb = cur.work_begin;
+    if (wb >= u1) break;
+    // this entry's quanta occupy units [wb + overhead, wb + gen_units)
+    const uint64_t q_base = wb + kGenEntryUnits;
+    const uint64_t lo = umax(u0, q_base), hi = umin(u1, wb + gen_units(cur.s));
+    if (hi <= lo) continue;
     if (threadIdx.x == 0) ctx = make_ctx(cur.s, p.arena);
     __syncthreads();
-    const syn_spec& s = cur.s;
-    const uint64_t tend = umin(t1, cur.tile_begin + gen_tiles(s));
-    if (tend > t) {
-      const uint64_t i0 = (t - cur.tile_begin) * kGenTileElems;
-      const uint64_t i1 = umin((tend - cur.tile_begin) * kGenTileElems, s.n);
-      gen_run<DT, DIST, SV_GEN_QPI>(ctx, s, i0, i1, p.arena);
-      t = tend;
-    }
-    ++e;
+    const uint64_t i0 = (lo - q_base) * 4, i1 = umin((hi - q_base) * 4, cur.s.n);
+    gen_run<DT, DIST, SV_GEN_QPI>(ctx, cur.s, i0, i1, p.arena);
   }
 }
 
@@ -242,10 +239,10 @@ __device__ void fix_dispatch(const Ctx& c, const syn_spec& s, uint64_t u, uint8_
 __global__ void __launch_bounds__(kThreads) fixup_kernel(const __grid_constant__ GenParams p) {
   const uint64_t u = (uint64_t)blockIdx.x * kThreads + threadIdx.x;
   if (u >= p.total) return;
-  const DevSpec* e = entry(p, find_entry<true>(p, u));
+  const DevSpec* e = entry(p, find_fix_entry(p, u));
   const syn_spec s = e->s;
   const Ctx c = make_ctx(s, p.arena);
-  fix_dispatch(c, s, u - e->unit_begin, p.arena);
+  fix_dispatch(c, s, u - e->fix_begin, p.arena);
 }
 
 // ---------------------------------------------------------------------------
@@ -346,17 +343,17 @@ static void fill_params(GenParams& gp, const DevSpec* host, const DevSpec* dev, 
     for (int i = 0; i < n; ++i) gp.inl[i] = host[i];
 }
 
-LaunchShape generate_shape(uint32_t dtype, uint32_t dist, uint64_t tiles) {
+LaunchShape generate_shape(uint32_t dtype, uint32_t dist, uint64_t units, uint64_t tiles) {
   const void* k = gen_kernel_for(dtype, dist);
-  return shape_for(tiles, k ? grid_cap_for(k) : 1);
+  return shape_for(units, tiles, k ? grid_cap_for(k) : 1, (uint64_t)SV_GEN_QPI * kThreads);
 }
 
 cudaError_t launch_generate_group(uint32_t dtype, uint32_t dist, const DevSpec* host, const DevSpec* dev, int n,
-                                  uint64_t tiles, LaunchShape sh, uint8_t* arena, cudaStream_t st) {
-  if (tiles == 0 || n == 0) return cudaSuccess;
+                                  uint64_t units, LaunchShape sh, uint8_t* arena, cudaStream_t st) {
+  if (units == 0 || n == 0) return cudaSuccess;
   GenParams gp;
   fill_params(gp, host, dev, n);
-  gp.total = tiles;
+  gp.total = units;
   gp.chunk = sh.chunk;
   gp.arena = arena;
   switch (SV_COMBO(dtype, dist)) {

@@ -72,14 +72,15 @@ extern "C" int verify_compare_noalloc(const vc_pair* pairs, int n_pairs, const v
   struct Run {
     uint32_t dtype;
     int begin, end;
-    uint64_t tiles;
+    uint64_t tiles, units;
   };
   std::vector<Run> runs;
   for (int k = 0; k < n_pairs; ++k) {
     const vc_pair& p = pairs[order[k]];
-    if (runs.empty() || runs.back().dtype != p.dtype) runs.push_back(Run{p.dtype, k, k, 0});
+    if (runs.empty() || runs.back().dtype != p.dtype) runs.push_back(Run{p.dtype, k, k, 0, 0});
     runs.back().end = k + 1;
     runs.back().tiles += cmp_tiles(p);
+    runs.back().units += cmp_units(p);
   }
   uint64_t slots = 0;
   for (const Run& r : runs) slots += std::min<uint64_t>(r.tiles, kGridCap) + (uint64_t)(r.end - r.begin);
@@ -93,26 +94,26 @@ extern "C" int verify_compare_noalloc(const vc_pair* pairs, int n_pairs, const v
   uint64_t slot_base = 0;
   for (size_t g = 0; g < runs.size(); ++g) {
     const Run& r = runs[g];
-    shapes[g] = compare_shape(r.dtype, r.tiles);
+    shapes[g] = compare_shape(r.dtype, r.units, r.tiles);
     uint64_t t = 0;
     for (int k = r.begin; k < r.end; ++k) {
       DevPair& d = tab[k];
       d.p = pairs[order[k]];
-      d.tile_begin = t;
+      d.work_begin = t;
       d.chunk = shapes[g].chunk;
       d.slot0 = slot_base + (uint64_t)(k - r.begin);
       d.orig = (uint32_t)order[k];
       d.pad = 0;
-      t += cmp_tiles(d.p);
+      t += cmp_units(d.p);
     }
-    slot_base += shapes[g].grid + (uint64_t)(r.end - r.begin);
+    slot_base += shapes[g].grid + (uint64_t)(r.end - r.begin) - 1;  // slots slot0 + b, b < grid
   }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const uint8_t* cand = static_cast<const uint8_t*>(d_cand);
   const uint8_t* ref = static_cast<const uint8_t*>(d_ref);
   for (size_t g = 0; g < runs.size(); ++g) {
     const Run& r = runs[g];
-    if (launch_compare_group(r.dtype, tab + r.begin, nullptr, r.end - r.begin, r.tiles, shapes[g], cand, ref,
+    if (launch_compare_group(r.dtype, tab + r.begin, nullptr, r.end - r.begin, r.units, shapes[g], cand, ref,
                              scratch, nullptr, st) != cudaSuccess)
       return SV_ECUDA;
   }

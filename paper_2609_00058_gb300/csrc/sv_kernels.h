@@ -23,18 +23,26 @@ constexpr int kThreads = 256;              // threads per CTA of every kernel
 constexpr uint32_t kGenTileElems = 8192;   // elements per generator tile
 constexpr uint32_t kCmpTileBytes = 16384;  // bytes per operand per compare tile
 constexpr uint32_t kGridCap = 4096;        // most persistent CTAs per launch
+constexpr int kStagedStarts = 2048;        // tables up to this size are searched in shared memory
+
+// Work is scheduled in weighted units: every entry costs a fixed overhead
+// (staging it, building its context, flushing its statistics) plus its
+// elements, and each CTA of a persistent grid takes an equal contiguous slice
+// of the units, so many small entries spread as evenly as a few large ones.
+constexpr uint64_t kGenEntryUnits = 1024;  // generator: units are 4-element quanta
+constexpr uint64_t kCmpEntryUnits = 512;   // compare: units are 16-byte vectors
 
 // generator table entry: the caller's spec plus scheduling data
 struct DevSpec {
   syn_spec s;
-  uint64_t tile_begin;  // first tile inside its group's tile list
-  uint64_t unit_begin;  // first thread in the exact-count fixup's list
+  uint64_t work_begin;  // first unit inside its group's unit range
+  uint64_t fix_begin;   // first thread in the exact-count fixup's list
 };
 
 // compare table entry: the caller's pair plus scheduling data
 struct DevPair {
   vc_pair p;
-  uint64_t tile_begin;  // first tile inside its group's tile list
+  uint64_t work_begin;  // first unit inside its group's unit range
   uint64_t chunk;       // tiles per CTA of its group's launch
   uint64_t slot0;       // partial slot of CTA 0 for this pair (slot0 + b for CTA b)
   uint32_t orig;        // index of the pair in the caller's table (result slot)
@@ -56,8 +64,12 @@ struct LaunchShape {
   uint64_t chunk;  // tiles per CTA
 };
 
-// persistent grid for `tiles` tiles: at most `cap` CTAs, contiguous chunks
-LaunchShape shape_for(uint64_t tiles, uint32_t cap);
+// persistent grid over `units` weighted units: at most min(cap, tiles) CTAs
+// (tiles: 8192-element generator or 16 KiB compare tiles, which bounds the
+// grid and so the compare's partial slots), contiguous chunks of units
+// (align: the chunk is rounded up to a multiple of it, one loop iteration of
+// the kernel, so every slice starts on an iteration boundary)
+LaunchShape shape_for(uint64_t units, uint64_t tiles, uint32_t cap, uint64_t align);
 // SMs x resident CTAs of this kernel (cached per device), at most kGridCap
 uint32_t grid_cap_for(const void* kernel);
 
@@ -65,8 +77,16 @@ SV_HD inline uint64_t cmp_tiles(const vc_pair& p) {
   const uint64_t sz = p.dtype == SV_I64 ? 8 : ((p.dtype == SV_F16 || p.dtype == SV_BF16) ? 2 : 4);
   return (p.n * sz + kCmpTileBytes - 1) / kCmpTileBytes;
 }
+SV_HD inline uint64_t cmp_vectors(const vc_pair& p) {
+  const uint64_t sz = p.dtype == SV_I64 ? 8 : ((p.dtype == SV_F16 || p.dtype == SV_BF16) ? 2 : 4);
+  return (p.n * sz + 15) / 16;
+}
+SV_HD inline uint64_t cmp_units(const vc_pair& p) { return kCmpEntryUnits + cmp_vectors(p); }
 SV_HD inline uint64_t gen_tiles(const syn_spec& s) {
   return s.dist == SV_DOTLIKE ? 0 : (s.n + kGenTileElems - 1) / kGenTileElems;
+}
+SV_HD inline uint64_t gen_units(const syn_spec& s) {
+  return s.dist == SV_DOTLIKE ? 0 : kGenEntryUnits + (s.n + 3) / 4;
 }
 SV_HD inline uint64_t fix_units(const syn_spec& s) {
   if (s.cand_offset == SV_NO_OUTPUT) return 0;
@@ -75,17 +95,17 @@ SV_HD inline uint64_t fix_units(const syn_spec& s) {
 }
 
 // ---- generator ----
-LaunchShape generate_shape(uint32_t dtype, uint32_t dist, uint64_t tiles);
+LaunchShape generate_shape(uint32_t dtype, uint32_t dist, uint64_t units, uint64_t tiles);
 // entries: either host (n <= SV_INLINE_ENTRIES, copied into the launch) or device
 cudaError_t launch_generate_group(uint32_t dtype, uint32_t dist, const DevSpec* host, const DevSpec* dev, int n,
-                                  uint64_t tiles, LaunchShape sh, uint8_t* arena, cudaStream_t st);
+                                  uint64_t units, LaunchShape sh, uint8_t* arena, cudaStream_t st);
 cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_t units, uint8_t* arena,
                          cudaStream_t st);
 cudaError_t launch_dotlike(const DevSpec& spec, uint8_t* arena, cudaStream_t st);
 
 // ---- compare ----
-LaunchShape compare_shape(uint32_t dtype, uint64_t tiles);
-cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevPair* dev, int n, uint64_t tiles,
+LaunchShape compare_shape(uint32_t dtype, uint64_t units, uint64_t tiles);
+cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevPair* dev, int n, uint64_t units,
                                  LaunchShape sh, const uint8_t* cand, const uint8_t* ref, Partial* partials,
                                  const int32_t* flag, cudaStream_t st);
 cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const Partial* partials,
