@@ -99,6 +99,8 @@ static int check_spec(const syn_spec& s, uint64_t arena) {
   const uint32_t imask = SV_SP_ZERO | SV_SP_IMIN | SV_SP_IMAX | SV_SP_DUP;
   if (s.special_mask & ~(fl ? fmask : imask)) return SV_EINVAL;
   if (!valid_rate(s.special_rate)) return SV_EINVAL;
+  if ((s.dist == SV_UNIFORM || s.dist == SV_NORMAL) && !(std::isfinite(s.p0) && std::isfinite(s.p1)))
+    return SV_EINVAL;  // finite parameters keep every drawn value finite
   if (s.dist == SV_UNIFORM && !(s.p1 >= s.p0)) return SV_EINVAL;
   if (s.dist == SV_INT_RANGE) {
     if (s.i1 < s.i0) return SV_EINVAL;

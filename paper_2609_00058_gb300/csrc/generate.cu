@@ -60,7 +60,12 @@ __device__ __forceinline__ void store4(uint8_t* base, uint64_t i, const typename
     else for (uint32_t j = 0; j < valid; ++j) p[j] = (uint16_t)v[j];
   } else {
     uint64_t* p = reinterpret_cast<uint64_t*>(base) + i;
-    if (valid == 4) {
+    if (valid == 4 && (reinterpret_cast<uintptr_t>(p) & 31) == 0) {
+      // one 256-bit store: a warp writes 1 KiB contiguously in one instruction
+      // (two 128-bit stores would each cover every other 16 bytes of it)
+      asm volatile("st.global.v4.u64 [%0], {%1, %2, %3, %4};" ::"l"(p), "l"(v[0]), "l"(v[1]), "l"(v[2]), "l"(v[3])
+                   : "memory");
+    } else if (valid == 4) {
       reinterpret_cast<ulonglong2*>(p)[0] = make_ulonglong2(v[0], v[1]);
       reinterpret_cast<ulonglong2*>(p)[1] = make_ulonglong2(v[2], v[3]);
     } else {
@@ -93,13 +98,25 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
     T v[QPI][4];
     uint64_t qu[QPI];
 #pragma unroll
-    for (int u = 0; u < QPI; ++u) {
-      qu[u] = umin(q + (uint64_t)u * kThreads, q1 - 1);
-      base4<DT, DIST>(c, eo + (qu[u] << 2), v[u]);
-    }
-    if (c.sp_thr) {
+    for (int u = 0; u < QPI; ++u) qu[u] = umin(q + (uint64_t)u * kThreads, q1 - 1);
+    if (one_block_dist<DT, DIST>() && c.sp_thr) {
+      // the quantum's VALUE and SPECIAL_SEL blocks as two interleaved chains
 #pragma unroll
-      for (int u = 0; u < QPI; ++u) specials4<DT, DIST>(c, cold, eo + (qu[u] << 2), v[u]);
+      for (int u = 0; u < QPI; ++u) {
+        const uint64_t g = eo + (qu[u] << 2), blk = g >> 2;
+        uint4 wv = make_uint4((uint32_t)blk, (uint32_t)(blk >> 32), c.stream, P_VALUE);
+        uint4 ws = make_uint4((uint32_t)blk, (uint32_t)(blk >> 32), c.stream, P_SPECIAL_SEL);
+        philox2_rk(wv, ws, c.rk);
+        base4_words<DT, DIST>(c, wv, v[u]);
+        specials4_words<DT, DIST>(c, cold, g, ws, v[u]);
+      }
+    } else {
+#pragma unroll
+      for (int u = 0; u < QPI; ++u) base4<DT, DIST>(c, eo + (qu[u] << 2), v[u]);
+      if (c.sp_thr) {
+#pragma unroll
+        for (int u = 0; u < QPI; ++u) specials4<DT, DIST>(c, cold, eo + (qu[u] << 2), v[u]);
+      }
     }
 #pragma unroll
     for (int u = 0; u < QPI; ++u) {

@@ -77,6 +77,8 @@ BAD_SPECS = [
     (dict(specials=("nan",), special_rate=1.5), -1),               # rate above 1
     (dict(specials=("nan",), special_rate=float("nan")), -1),      # NaN rate
     (dict(p0=1.0, p1=-1.0), -1),                                   # empty uniform range
+    (dict(p0=float("-inf"), p1=1.0), -1),                          # infinite uniform bound
+    (dict(dist="normal", p0=0.0, p1=float("nan")), -1),            # non-finite normal scale
     (dict(logical_n=100), -1),                                     # n beyond the logical length
     (dict(logical_n=1 << 41), -3),                                 # logical length beyond the limit
     (dict(pelem=W.Perturb("count_set", count=1)), -1),             # count kind in the element-wise slot
