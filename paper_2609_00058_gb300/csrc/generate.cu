@@ -6,11 +6,14 @@
 //                 then the clean output and (after the element-wise
 //                 perturbation) the perturbed twin, as 16-byte stores.
 //   fixup_kernel  one thread per exact-count edit (or swapped pair).
-//   dot_kernel    64 x 128 output tiles of the dot-like values with the
-//                 factors staged in shared memory; same epilogue per quantum.
+//   dot_kernel    persistent; 64 x 128 output tiles of the dot-like values,
+//                 factors streamed through shared memory by cp.async; same
+//                 epilogue per quantum.
 //
 // Bound: HBM writes for cheap maps; the Philox/Box-Muller ALU work for
 // normals; FP32 FMA for the dot-like values.
+#include <algorithm>
+
 #include "sv_device.cuh"
 #include "sv_kernels.h"
 
@@ -263,91 +266,196 @@ __global__ void __launch_bounds__(kThreads) fixup_kernel(const __grid_constant__
 }
 
 // ---------------------------------------------------------------------------
-// dot-like values: 64 x 128 output tile per CTA, 8 rows x 4 columns per thread
-// (one quantum per row), factors staged in shared memory 32 k at a time; each
-// output is the k-ascending chain of fused multiply-adds.
+// dot-like values: persistent CTAs, each a contiguous run of 64 x 128 output
+// tiles (row-block major, so consecutive tiles share their A rows).  The
+// factors stream through a ring of kDotStages shared-memory slots, one
+// 32-deep k chunk of A (64 rows x 32, row-major) and B (32 x 128) per slot,
+// filled by cp.async while earlier chunks are multiplied; every output is the
+// k-ascending chain of fused multiply-adds over exactly its K steps.  Thread
+// layout: warp w owns rows 8w..8w+7 of the tile, lane l columns 4l..4l+3 (one
+// quantum per row), so a warp's A reads are broadcasts and its B reads and
+// output stores are contiguous.
 // ---------------------------------------------------------------------------
-constexpr int kDotRows = 64, kDotCols = 128, kDotK = 32, kDotPad = 4;
+#ifndef SV_DOT_STAGES
+#define SV_DOT_STAGES 3
+#endif
+#ifndef SV_DOT_MINB
+#define SV_DOT_MINB 2
+#endif
+constexpr int kDotRows = 64, kDotCols = 128, kDotK = 32, kDotStages = SV_DOT_STAGES;
+constexpr int kDotSlotFloats = kDotRows * kDotK + kDotK * kDotCols;
+constexpr size_t kDotSmem = (size_t)kDotStages * kDotSlotFloats * sizeof(float);
 
 struct DotParams {
   DevSpec spec;
   uint8_t* arena;
-  uint64_t row0;  // first row of the chunk
+  uint64_t row0;   // first row of the chunk
+  uint64_t tiles;  // row blocks x column blocks
+  uint32_t n_cb;   // column blocks
 };
 
-template <int DT>
-__global__ void __launch_bounds__(kThreads) dot_kernel(const __grid_constant__ DotParams p) {
+__device__ __forceinline__ void cp_async16(float* dst, const float* src, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(src), "r"(valid ? 16 : 0) : "memory");
+}
+__device__ __forceinline__ void cp_async4(float* dst, const float* src, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(src), "r"(valid ? 4 : 0) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+// position in a CTA's run of (tile, k chunk) steps, advanced without division
+struct DotCursor {
+  uint64_t rb, cb, kc;  // row block (relative to row0), column block, first k of the chunk
+  __device__ __forceinline__ void advance(uint64_t K, uint32_t n_cb) {
+    kc += kDotK;
+    if (kc >= K) {
+      kc = 0;
+      if (++cb == n_cb) cb = 0, ++rb;
+    }
+  }
+};
+
+// A16: the A rows are 16-byte aligned (K % 4 == 0) and move in 16-byte pieces
+template <int DT, bool A16>
+__global__ void __launch_bounds__(kThreads, SV_DOT_MINB) dot_kernel(const __grid_constant__ DotParams p) {
   using T = typename Store<DT>::T;
-  __shared__ __align__(16) float As[kDotK][kDotRows + kDotPad];  // A transposed: [k][row]
-  __shared__ __align__(16) float Bs[kDotK][kDotCols];
+  extern __shared__ __align__(128) float dsm[];
   __shared__ Ctx cold;
   const syn_spec& s = p.spec.s;
   if (threadIdx.x == 0) cold = make_ctx(s, p.arena);
   __syncthreads();
   const Ctx c = cold;
   const uint64_t rows = s.rows, cols = s.cols, K = s.dot_k;
-  const uint64_t r0 = p.row0 + (uint64_t)blockIdx.y * kDotRows;
-  const uint64_t c0 = (uint64_t)blockIdx.x * kDotCols;
   const int tid = threadIdx.x, cg = tid & 31, rg = tid >> 5;
+  const uint64_t t_begin = p.tiles * blockIdx.x / gridDim.x, t_end = p.tiles * (blockIdx.x + 1) / gridDim.x;
+  const uint64_t nk = (K + kDotK - 1) / kDotK;
+  const uint64_t steps = (t_end - t_begin) * nk;
+  const DotCursor first{t_begin / p.n_cb, t_begin % p.n_cb, 0};
+
+  // step i of this CTA goes to slot i % kDotStages; the copy of step i is
+  // issued at iteration i - (kDotStages - 1), so `ic` runs that far ahead
+  DotCursor ic = first;
+  uint64_t issued = 0;
+  uint32_t islot = 0;
+  auto issue = [&]() {
+    if (issued < steps) {
+      const uint64_t r0 = p.row0 + ic.rb * kDotRows, c0 = ic.cb * kDotCols, kc = ic.kc;
+      float* As = dsm + islot * kDotSlotFloats;
+      float* Bs = As + kDotRows * kDotK;
+      if constexpr (A16) {
+#pragma unroll
+        for (int it = 0; it < kDotRows * kDotK / 4 / kThreads; ++it) {
+          const int r = (tid >> 3) + it * (kThreads / 8), q = tid & 7;
+          const uint64_t gr = r0 + r, gk = kc + 4 * q;
+          const bool ok = gr < rows && gk < K;  // K % 4 == 0: the whole piece is in range
+          cp_async16(As + r * kDotK + 4 * q, ok ? c.A + gr * K + gk : c.A, ok);
+        }
+      } else {
+#pragma unroll
+        for (int it = 0; it < kDotRows * kDotK / kThreads; ++it) {
+          const int r = (tid >> 5) + it * (kThreads / 32), k = tid & 31;
+          const uint64_t gr = r0 + r, gk = kc + k;
+          const bool ok = gr < rows && gk < K;
+          cp_async4(As + r * kDotK + k, ok ? c.A + gr * K + gk : c.A, ok);
+        }
+      }
+#pragma unroll
+      for (int it = 0; it < kDotK * kDotCols / 4 / kThreads; ++it) {
+        const int k = (tid >> 5) + it * (kThreads / 32), q = tid & 31;
+        const uint64_t gk = kc + k, gc = c0 + 4 * q;
+        const bool ok = gk < K && gc < cols;  // cols % 4 == 0
+        cp_async16(Bs + k * kDotCols + 4 * q, ok ? c.B + gk * cols + gc : c.B, ok);
+      }
+      ic.advance(K, p.n_cb);
+      ++issued;
+      islot = islot + 1 == kDotStages ? 0 : islot + 1;
+    }
+    cp_async_commit();  // one group per step, empty past the end: uniform counting
+  };
+
+  for (int i = 0; i < kDotStages - 1; ++i) issue();
+
+  uint8_t* ref = s.ref_offset == SV_NO_OUTPUT ? nullptr : p.arena + s.ref_offset;
+  uint8_t* cand = s.cand_offset == SV_NO_OUTPUT ? nullptr : p.arena + s.cand_offset;
+  const uint64_t lo = s.elem_offset, hi = s.elem_offset + s.n;
   float acc[8][4];
 #pragma unroll
   for (int r = 0; r < 8; ++r)
 #pragma unroll
     for (int j = 0; j < 4; ++j) acc[r][j] = 0.0f;
 
-  for (uint64_t kc = 0; kc < K; kc += kDotK) {
-    const int kn = (int)umin(kDotK, K - kc);
-    __syncthreads();
-    for (int l = tid; l < kDotRows * kDotK; l += kThreads) {  // A tile, rows x k
-      const int r = l / kDotK, k = l % kDotK;
-      const uint64_t gr = r0 + r;
-      As[k][r] = (gr < rows && k < kn) ? c.A[gr * K + kc + k] : 0.0f;
-    }
-    for (int l = tid; l < kDotK * (kDotCols / 4); l += kThreads) {  // B tile, k x cols
-      const int k = l / (kDotCols / 4), q = l % (kDotCols / 4);
-      const uint64_t gc = c0 + 4 * q;
-      float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (k < kn && gc < cols) b = *reinterpret_cast<const float4*>(c.B + (kc + k) * cols + gc);
-      *reinterpret_cast<float4*>(&Bs[k][4 * q]) = b;
-    }
-    __syncthreads();
-    for (int k = 0; k < kn; ++k) {
-      const float4 a0 = *reinterpret_cast<const float4*>(&As[k][8 * rg]);
-      const float4 a1 = *reinterpret_cast<const float4*>(&As[k][8 * rg + 4]);
-      const float4 b = *reinterpret_cast<const float4*>(&Bs[k][4 * cg]);
-      const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-      const float bb[4] = {b.x, b.y, b.z, b.w};
+  DotCursor cc = first;
+  uint32_t cslot = 0;
+  for (uint64_t i = 0; i < steps; ++i) {
+    cp_async_wait<kDotStages - 2>();
+    __syncthreads();  // chunk i landed for every thread; slot (i - 1) % kDotStages is free
+    issue();
+    const float* As = dsm + cslot * kDotSlotFloats + (8 * rg) * kDotK;
+    const float* Bs = dsm + cslot * kDotSlotFloats + kDotRows * kDotK + 4 * cg;
+    cslot = cslot + 1 == kDotStages ? 0 : cslot + 1;
+    const int kn = (int)umin(kDotK, K - cc.kc);
+    int k = 0;
+    for (; k + 4 <= kn; k += 4) {
+      float4 a[8], b[4];
 #pragma unroll
-      for (int r = 0; r < 8; ++r)
+      for (int r = 0; r < 8; ++r) a[r] = *reinterpret_cast<const float4*>(As + r * kDotK + k);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[r][j] = __fmaf_rn(a[r], bb[j], acc[r][j]);
+      for (int q = 0; q < 4; ++q) b[q] = *reinterpret_cast<const float4*>(Bs + (k + q) * kDotCols);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+          const float ar = q == 0 ? a[r].x : q == 1 ? a[r].y : q == 2 ? a[r].z : a[r].w;
+          acc[r][0] = __fmaf_rn(ar, b[q].x, acc[r][0]);
+          acc[r][1] = __fmaf_rn(ar, b[q].y, acc[r][1]);
+          acc[r][2] = __fmaf_rn(ar, b[q].z, acc[r][2]);
+          acc[r][3] = __fmaf_rn(ar, b[q].w, acc[r][3]);
+        }
+      }
     }
-  }
+    for (; k < kn; ++k) {  // K % 4 != 0: exactly the remaining steps, no zero padding
+      const float4 b = *reinterpret_cast<const float4*>(Bs + k * kDotCols);
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        const float ar = As[r * kDotK + k];
+        acc[r][0] = __fmaf_rn(ar, b.x, acc[r][0]);
+        acc[r][1] = __fmaf_rn(ar, b.y, acc[r][1]);
+        acc[r][2] = __fmaf_rn(ar, b.z, acc[r][2]);
+        acc[r][3] = __fmaf_rn(ar, b.w, acc[r][3]);
+      }
+    }
+    const DotCursor at = cc;
+    cc.advance(K, p.n_cb);
+    if (cc.kc != 0) continue;  // the tile has more k chunks
 
-  uint8_t* ref = s.ref_offset == SV_NO_OUTPUT ? nullptr : p.arena + s.ref_offset;
-  uint8_t* cand = s.cand_offset == SV_NO_OUTPUT ? nullptr : p.arena + s.cand_offset;
-  const uint64_t col = c0 + 4 * cg;
-  if (col >= cols) return;
-  const uint64_t lo = s.elem_offset, hi = s.elem_offset + s.n;
+    // epilogue of the tile: rounding, specials, clean store, perturbation, twin store
+    const uint64_t r0 = p.row0 + at.rb * kDotRows, col = at.cb * kDotCols + 4 * cg;
 #pragma unroll
-  for (int r = 0; r < 8; ++r) {
-    const uint64_t row = r0 + 8 * rg + r;
-    if (row >= rows) break;
-    const uint64_t g = row * cols + col;  // multiple of 4 (cols % 4 == 0)
-    if (g + 4 <= lo || g >= hi) continue;
-    T v[4];
+    for (int r = 0; r < 8; ++r) {
+      const uint64_t row = r0 + 8 * rg + r;
+      const uint64_t g = row * cols + col;  // multiple of 4 (cols % 4 == 0)
+      if (col < cols && row < rows && g + 4 > lo && g < hi) {
+        T v[4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) v[j] = (T)from_f32<DT>(acc[r][j]);
-    if (c.sp_thr) specials4<DT, SV_DOTLIKE>(c, cold, g, v);
-    // chunk bounds fall on quanta (elem_offset % 4 == 0); n may end mid-quantum
-    const uint64_t i = g - lo;
-    const uint32_t valid = (uint32_t)umin(4, hi - g);
-    if (ref) store4<DT>(ref, i, v, valid);
-    if (cand) {
-      if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, cold, g, v);
-      store4<DT>(cand, i, v, valid);
+        for (int j = 0; j < 4; ++j) v[j] = (T)from_f32<DT>(acc[r][j]);
+        if (c.sp_thr) specials4<DT, SV_DOTLIKE>(c, cold, g, v);
+        // chunk bounds fall on quanta (elem_offset % 4 == 0); n may end mid-quantum
+        const uint64_t e = g - lo;
+        const uint32_t valid = (uint32_t)umin(4, hi - g);
+        if (ref) store4<DT>(ref, e, v, valid);
+        if (cand) {
+          if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, cold, g, v);
+          store4<DT>(cand, e, v, valid);
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) acc[r][j] = 0.0f;
     }
   }
+  cp_async_wait<0>();
 }
 
 // ---------------------------------------------------------------------------
@@ -396,6 +504,15 @@ cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_
   return cudaGetLastError();
 }
 
+template <int DT, bool A16>
+static cudaError_t launch_dot(const DotParams& dp, uint64_t tiles, cudaStream_t st) {
+  const void* fn = reinterpret_cast<const void*>(dot_kernel<DT, A16>);
+  const uint32_t cap = grid_cap_for(fn, kDotSmem);
+  const unsigned grid = (unsigned)std::min<uint64_t>(tiles, cap);
+  dot_kernel<DT, A16><<<grid, kThreads, kDotSmem, st>>>(dp);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_dotlike(const DevSpec& spec, uint8_t* arena, cudaStream_t st) {
   const syn_spec& s = spec.s;
   if (s.n == 0) return cudaSuccess;
@@ -404,14 +521,14 @@ cudaError_t launch_dotlike(const DevSpec& spec, uint8_t* arena, cudaStream_t st)
   dp.arena = arena;
   const uint64_t first_row = s.elem_offset / s.cols, last_row = (s.elem_offset + s.n - 1) / s.cols;
   dp.row0 = first_row;
-  const dim3 grid((unsigned)((s.cols + kDotCols - 1) / kDotCols),
-                  (unsigned)((last_row - first_row + 1 + kDotRows - 1) / kDotRows));
+  dp.n_cb = (uint32_t)((s.cols + kDotCols - 1) / kDotCols);
+  dp.tiles = (last_row - first_row + kDotRows) / kDotRows * dp.n_cb;
+  const bool a16 = s.dot_k % 4 == 0;
   switch (s.dtype) {
-    case SV_F32: dot_kernel<SV_F32><<<grid, kThreads, 0, st>>>(dp); break;
-    case SV_F16: dot_kernel<SV_F16><<<grid, kThreads, 0, st>>>(dp); break;
-    default: dot_kernel<SV_BF16><<<grid, kThreads, 0, st>>>(dp); break;
+    case SV_F32: return a16 ? launch_dot<SV_F32, true>(dp, dp.tiles, st) : launch_dot<SV_F32, false>(dp, dp.tiles, st);
+    case SV_F16: return a16 ? launch_dot<SV_F16, true>(dp, dp.tiles, st) : launch_dot<SV_F16, false>(dp, dp.tiles, st);
+    default: return a16 ? launch_dot<SV_BF16, true>(dp, dp.tiles, st) : launch_dot<SV_BF16, false>(dp, dp.tiles, st);
   }
-  return cudaGetLastError();
 }
 
 }  // namespace sv

@@ -71,7 +71,7 @@ struct LaunchShape {
 // the kernel, so every slice starts on an iteration boundary)
 LaunchShape shape_for(uint64_t units, uint64_t tiles, uint32_t cap, uint64_t align);
 // SMs x resident CTAs of this kernel (cached per device), at most kGridCap
-uint32_t grid_cap_for(const void* kernel);
+uint32_t grid_cap_for(const void* kernel, size_t dyn_smem = 0);
 
 SV_HD inline uint64_t cmp_tiles(const vc_pair& p) {
   const uint64_t sz = p.dtype == SV_I64 ? 8 : ((p.dtype == SV_F16 || p.dtype == SV_BF16) ? 2 : 4);

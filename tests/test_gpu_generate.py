@@ -225,6 +225,21 @@ def test_dotlike_f32_and_odd_shapes(dev):
         assert np.array_equal(g, h), (rows, cols, k)
 
 
+def test_dotlike_many_tiles_per_cta(dev):
+    # more 64 x 128 tiles than resident CTAs, ragged in rows and columns, with
+    # K a multiple of 4 (16-byte factor rows) and not (4-byte factor copies)
+    for dtype, rows, cols, k in (("f16", 1100, 4100, 37), ("bf16", 1031, 4108, 68)):
+        ar = W.Arena()
+        ao, bo = ar.take(4 * rows * k), ar.take(4 * k * cols)
+        ro = ar.take(2 * rows * cols)
+        fa = W.GenSpec("f32", "uniform", rows * k, seed=5, stream=0, ref_offset=ao, p0=-1, p1=1)
+        fb = W.GenSpec("f32", "uniform", k * cols, seed=5, stream=1, ref_offset=bo, p0=-1, p1=1)
+        d = W.GenSpec(dtype, "dotlike", rows * cols, seed=5, stream=2, ref_offset=ro, rows=rows, cols=cols, dot_k=k,
+                      a_offset=ao, b_offset=bo, specials=("pinf", "zero"), special_rate=1e-3)
+        g, h = gen_both(dev, [[fa, fb], [d]], ar.size)
+        assert np.array_equal(g, h), (dtype, rows, cols, k)
+
+
 def test_dotlike_chunked(dev):
     rows, cols, k = 40, 64, 16
     ar = W.Arena()
