@@ -78,13 +78,19 @@ def alu_peaks():
 def alu_floor_s(wl, peaks):
     """Seconds the generator needs at the measured ALU rates: per 4-element
     quantum, its Philox blocks (value, special selection, element-wise
-    perturbation) and Box-Muller pairs (normal values, noise)."""
+    perturbation) and Box-Muller pairs (normal values, noise); for dot-like
+    values also the K fp32 FMAs of every output."""
     cycles = 0.0
     for call in wl.gen_calls:
         for s in call:
-            if s.dist == "dotlike":
-                return None
             quanta = (s.n + 3) // 4
+            if s.dist == "dotlike":  # K fp32 FMAs per output, then the same per-quantum noise
+                cycles += 4 * quanta * s.dot_k / peaks["ffma_per_sm_cycle"]
+                blocks = 1 if s.pelem.kind in ("rate_add_pm", "rel_noise") and s.cand_offset is not None else 0
+                pairs = 2 if s.pelem.kind == "rel_noise" else 0
+                cycles += quanta * (blocks / peaks["philox_blocks_per_sm_cycle"] +
+                                    pairs / peaks["box_muller_pairs_per_sm_cycle"])
+                continue
             blocks = {"uniform": 1, "normal": 1, "int_range": 2 if s.dtype == "i64" else 1,
                       "raw_bits": 2 if s.dtype == "i64" else 1}.get(s.dist, 0)
             blocks += 1 if s.specials and s.special_rate > 0 else 0
@@ -357,10 +363,10 @@ def ours_arm(args, rank, world):
         alu_gbs = gen_bytes_launch / alu_s / 1e9
         roofline = {"bound": "alu", "kernel": "syn_generate (gen_kernel + exact-count fixup)",
                     "achieved": achieved, "peak": alu_gbs, "unit": "GB/s", "frac": achieved / alu_gbs,
-                    "peak_kind": "measured ALU rates (Philox %.3f blocks, Box-Muller %.3f pairs per SM-cycle, "
-                                 "%d SMs at %d MHz) as output GB/s" % (alu["philox_blocks_per_sm_cycle"],
-                                                                      alu["box_muller_pairs_per_sm_cycle"],
-                                                                      alu["sms"], alu["clock_mhz"]),
+                    "peak_kind": "measured ALU rates (Philox %.3f blocks, Box-Muller %.3f pairs, %.1f fp32 FMAs "
+                                 "per SM-cycle, %d SMs at %d MHz) as output GB/s" % (
+                                     alu["philox_blocks_per_sm_cycle"], alu["box_muller_pairs_per_sm_cycle"],
+                                     alu["ffma_per_sm_cycle"], alu["sms"], alu["clock_mhz"]),
                     "hbm_peak": hbm, "hbm_frac": achieved / hbm, "traffic": traffic}
     else:
         roofline = {"bound": "hbm", "kernel": "syn_generate (gen_kernel + exact-count fixup)",

@@ -54,6 +54,52 @@ __global__ void box_muller_kernel(uint32_t* out) {
   if (acc == 12345.0f) out[t] = 1;
 }
 
+// fp32 fused multiply-adds, scalar and packed pairs (fma.rn.f32x2): 16
+// independent accumulators per thread, counted in single FMAs
+__global__ void ffma_kernel(float* out, float x) {
+  float acc[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) acc[j] = (float)(threadIdx.x + j);
+  const float y = x * 0.5f;
+  for (int i = 0; i < kIter; i += 16) {
+#pragma unroll
+    for (int u = 0; u < 16; ++u)
+#pragma unroll
+      for (int j = 0; j < 16; ++j) acc[j] = __fmaf_rn(acc[j], x, y);
+  }
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) s += acc[j];
+  if (s == 12345.0f) out[threadIdx.x] = s;
+}
+
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+
+__global__ void ffma2_kernel(float* out, float x) {
+  uint64_t acc[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const float lo = (float)(threadIdx.x + j), hi = (float)(threadIdx.x + 2 * j);
+    acc[j] = ((uint64_t)__float_as_uint(hi) << 32) | __float_as_uint(lo);
+  }
+  const uint64_t xx = ((uint64_t)__float_as_uint(x) << 32) | __float_as_uint(x);
+  const uint64_t yy = ((uint64_t)__float_as_uint(x * 0.5f) << 32) | __float_as_uint(x * 0.5f);
+  for (int i = 0; i < kIter; i += 16) {
+#pragma unroll
+    for (int u = 0; u < 16; ++u)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[j] = fma2(acc[j], xx, yy);
+  }
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) s += __uint_as_float((uint32_t)acc[j]) + __uint_as_float((uint32_t)(acc[j] >> 32));
+  if (s == 12345.0f) out[threadIdx.x] = s;
+}
+
 template <class F>
 double per_sm_cycle(F launch, double units, int sms, int clk_khz) {
   cudaEvent_t a, b;
@@ -82,9 +128,13 @@ int main() {
   const double work = (double)blocks * threads * kIter;
   const double philox = per_sm_cycle([&] { philox_kernel<<<blocks, threads>>>(out, 1, 2); }, work, sms, clk);
   const double bm = per_sm_cycle([&] { box_muller_kernel<<<blocks, threads>>>(out); }, work, sms, clk);
+  float* fout = reinterpret_cast<float*>(out);
+  const double ffma = per_sm_cycle([&] { ffma_kernel<<<blocks, threads>>>(fout, 0.999f); }, work * 16, sms, clk);
+  const double ffma2 = per_sm_cycle([&] { ffma2_kernel<<<blocks, threads>>>(fout, 0.999f); }, work * 16, sms, clk);
   cudaFree(out);
   if (cudaGetLastError() != cudaSuccess) return 1;
-  printf("{\"philox_blocks_per_sm_cycle\": %.4f, \"box_muller_pairs_per_sm_cycle\": %.4f, \"sms\": %d, "
-         "\"clock_mhz\": %d}\n", philox, bm, sms, clk / 1000);
+  printf("{\"philox_blocks_per_sm_cycle\": %.4f, \"box_muller_pairs_per_sm_cycle\": %.4f, "
+         "\"ffma_per_sm_cycle\": %.2f, \"ffma2_fmas_per_sm_cycle\": %.2f, \"sms\": %d, \"clock_mhz\": %d}\n",
+         philox, bm, ffma, ffma2, sms, clk / 1000);
   return 0;
 }
