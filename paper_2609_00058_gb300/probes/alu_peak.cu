@@ -11,6 +11,7 @@
 namespace {
 constexpr uint32_t kM0 = 0xD2511F53u, kM1 = 0xCD9E8D57u, kW0 = 0x9E3779B9u, kW1 = 0xBB67AE85u;
 constexpr int kIter = 256;
+constexpr int kFmaIter = 4096;  // long enough (about 0.5 ms a launch) for a steady clock
 
 __device__ __forceinline__ uint4 block(uint4 c, uint32_t k0, uint32_t k1) {
 #pragma unroll
@@ -61,7 +62,7 @@ __global__ void ffma_kernel(float* out, float x) {
 #pragma unroll
   for (int j = 0; j < 16; ++j) acc[j] = (float)(threadIdx.x + j);
   const float y = x * 0.5f;
-  for (int i = 0; i < kIter; i += 16) {
+  for (int i = 0; i < kFmaIter; i += 16) {
 #pragma unroll
     for (int u = 0; u < 16; ++u)
 #pragma unroll
@@ -88,7 +89,7 @@ __global__ void ffma2_kernel(float* out, float x) {
   }
   const uint64_t xx = ((uint64_t)__float_as_uint(x) << 32) | __float_as_uint(x);
   const uint64_t yy = ((uint64_t)__float_as_uint(x * 0.5f) << 32) | __float_as_uint(x * 0.5f);
-  for (int i = 0; i < kIter; i += 16) {
+  for (int i = 0; i < kFmaIter; i += 16) {
 #pragma unroll
     for (int u = 0; u < 16; ++u)
 #pragma unroll
@@ -129,8 +130,9 @@ int main() {
   const double philox = per_sm_cycle([&] { philox_kernel<<<blocks, threads>>>(out, 1, 2); }, work, sms, clk);
   const double bm = per_sm_cycle([&] { box_muller_kernel<<<blocks, threads>>>(out); }, work, sms, clk);
   float* fout = reinterpret_cast<float*>(out);
-  const double ffma = per_sm_cycle([&] { ffma_kernel<<<blocks, threads>>>(fout, 0.999f); }, work * 16, sms, clk);
-  const double ffma2 = per_sm_cycle([&] { ffma2_kernel<<<blocks, threads>>>(fout, 0.999f); }, work * 16, sms, clk);
+  const double fwork = (double)blocks * threads * kFmaIter * 16;
+  const double ffma = per_sm_cycle([&] { ffma_kernel<<<blocks, threads>>>(fout, 0.999f); }, fwork, sms, clk);
+  const double ffma2 = per_sm_cycle([&] { ffma2_kernel<<<blocks, threads>>>(fout, 0.999f); }, fwork, sms, clk);
   cudaFree(out);
   if (cudaGetLastError() != cudaSuccess) return 1;
   printf("{\"philox_blocks_per_sm_cycle\": %.4f, \"box_muller_pairs_per_sm_cycle\": %.4f, "
