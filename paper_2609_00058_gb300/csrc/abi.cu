@@ -18,7 +18,7 @@ static_assert(sizeof(syn_spec) == 224, "syn_spec layout");
 static_assert(sizeof(vc_pair) == 48, "vc_pair layout");
 static_assert(sizeof(vc_result) == 80, "vc_result layout");
 static_assert(sizeof(Partial) == 64, "partial record layout");
-static_assert(sizeof(DevSpec) == 240, "spec table entry layout");
+static_assert(sizeof(DevSpec) == 248, "spec table entry layout");
 static_assert(sizeof(DevPair) == 80, "pair table entry layout");
 
 constexpr size_t kAlign = 256;
@@ -300,18 +300,35 @@ int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena
   std::vector<Group> groups;
   group_by(n_specs, [&](int i) { return specs[i].dtype * 8u + specs[i].dist; }, order, groups);
   std::vector<DevSpec> tab(n_specs);
-  uint64_t fixes = 0;
   for (Group& g : groups) {
     for (int k = g.begin; k < g.end; ++k) {
       const syn_spec& s = specs[order[k]];
       tab[k].s = s;
       tab[k].work_begin = g.units;
-      tab[k].fix_begin = fixes;
+      tab[k].fused = 0;
+      tab[k].pad = 0;
       g.units += gen_units(s);
       g.tiles += gen_tiles(s);
-      fixes += fix_units(s);
     }
     if (g.units) g.sh = generate_shape(tab[g.begin].s.dtype, tab[g.begin].s.dist, g.units, g.tiles);
+  }
+  // exact-count edits: applied by the generating CTAs where a CTA's slice (at
+  // most 4 x chunk elements) meets few strata, else by the fixup kernel
+  uint64_t fixes = 0;
+  for (const Group& g : groups) {
+    for (int k = g.begin; k < g.end; ++k) {
+      DevSpec& d = tab[k];
+      d.fix_begin = fixes;
+      const uint64_t units = fix_units(d.s);
+      if (units == 0) continue;
+      const uint64_t N = d.s.logical_n ? d.s.logical_n : d.s.elem_offset + d.s.n;
+      if (d.s.dist != SV_DOTLIKE && 4 * g.sh.chunk / N * fix_strata(d.s) +
+                                            (4 * g.sh.chunk % N) * fix_strata(d.s) / N + 2 <= kMaxFusedEdits) {
+        d.fused = 1;
+        continue;
+      }
+      fixes += units;
+    }
   }
   const DevSpec* dev = nullptr;
   if (need) {

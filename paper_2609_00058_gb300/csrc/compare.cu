@@ -412,6 +412,7 @@ __device__ vc_result fold_pair(const DevPair& dp, const Partial* partials, int l
   {
     // every CTA whose unit slice overlaps [work_begin, work_begin + units)
     const uint64_t b0 = dp.work_begin / dp.chunk, b1 = (dp.work_begin + cmp_units(pr) - 1) / dp.chunk;
+#pragma unroll 4  // independent record loads in flight together
     for (uint64_t b = b0 + lane; b <= b1; b += 32) {
       const Partial q = partials[dp.slot0 + b];
       mism += q.mism;

@@ -84,6 +84,63 @@ __device__ __forceinline__ void store4(uint8_t* base, uint64_t i, const typename
 #define SV_GEN_MINB 2  // resident CTAs per SM the register budget must allow
 #endif
 
+// ---------------------------------------------------------------------------
+// exact-count perturbations: the index of stratum st of [0, N) cut into k
+// strata is floor(st N / k) + mulhi64(x, len), x from INDEX block st; a
+// COUNT edit sets or offsets the candidate value there, SWAP_PAIRS exchanges
+// the candidate values of strata 2j and 2j + 1.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t stratum_index(const Ctx& c, uint32_t stream, uint64_t k, uint64_t st) {
+  const uint64_t start = (st * c.N) / k, end = ((st + 1) * c.N) / k;  // st < 2^21, N <= 2^40
+  const uint4 w = draw(c.rk, stream, P_INDEX, st);
+  const uint64_t x = ((uint64_t)w.x << 32) | w.y;
+  return start + __umul64hi(x, end - start);
+}
+
+// the stratum holding logical index g: the largest st with floor(st N / k) <= g
+__device__ __forceinline__ uint64_t stratum_of(uint64_t g, uint64_t k, uint64_t N) {
+  return umin(((g + 1) * k - 1) / N, k - 1);  // (g + 1) k < 2^61
+}
+
+// candidate bits at g after a COUNT_SET / COUNT_ADD edit
+template <int DT, int DIST>
+__device__ uint64_t count_edit_bits(const Ctx& c, const sv_perturb& pc, uint64_t g) {
+  const uint64_t v2 = value_at<DT, DIST>(c, g, 1);
+  if constexpr (is_float(DT)) {
+    const float f = __double2float_rn(pc.value);
+    if (pc.kind == SV_PERT_COUNT_SET) return from_f32<DT>(f);
+    const uint32_t b = (uint32_t)v2;
+    return finite_bits<DT>(b) ? from_f32<DT>(__fadd_rn(to_f32<DT>(b), f)) : from_f32<DT>(f);
+  } else {
+    return pc.kind == SV_PERT_COUNT_SET ? ((uint64_t)pc.ivalue & width_mask(DT))
+                                        : ((v2 + (uint64_t)pc.ivalue) & width_mask(DT));
+  }
+}
+
+// the edits of the strata that meet logical range [g0, g1), which this CTA
+// has just generated: thread t < m takes stratum sf + t and overwrites the
+// candidate element if the stratum's index falls in the range (m <=
+// kMaxFusedEdits, which the host guarantees for fused specs).  The caller's
+// __syncthreads() orders these stores after the CTA's own generating stores;
+// no other CTA writes [g0, g1).  The values equal what the fixup kernel writes.
+template <int DT, int DIST>
+__device__ __noinline__ void fused_edits(const Ctx& c, const syn_spec& s, uint64_t g0, uint64_t g1, uint8_t* arena) {
+  using T = typename Store<DT>::T;
+  const sv_perturb& pc = s.pcount;
+  const uint64_t k = fix_strata(s);
+  const uint64_t sf = stratum_of(g0, k, c.N), sl = stratum_of(g1 - 1, k, c.N);
+  const uint64_t m = umin(sl - sf + 1, kMaxFusedEdits);
+  if (threadIdx.x >= m) return;
+  const uint64_t st = sf + threadIdx.x;
+  const uint64_t g = stratum_index(c, pc.stream, k, st);
+  if (g < g0 || g >= g1) return;
+  const uint64_t bits = pc.kind == SV_PERT_SWAP_PAIRS ? value_at<DT, DIST>(c, stratum_index(c, pc.stream, k, st ^ 1), 1)
+                                                      : count_edit_bits<DT, DIST>(c, pc, g);
+  uint8_t* cand = arena + s.cand_offset;
+  if constexpr (elem_bytes(DT) == 2) reinterpret_cast<uint16_t*>(cand)[g - s.elem_offset] = (uint16_t)bits;
+  else reinterpret_cast<T*>(cand)[g - s.elem_offset] = (T)bits;
+}
+
 // elements [i0, i1) of one spec, by 4-element quanta spread over the CTA.
 // `cold` is the spec's context in shared memory; the hot fields are copied to
 // registers.  Each thread carries QPI quanta at once so their Philox and
@@ -161,6 +218,10 @@ __global__ void __launch_bounds__(kThreads, SV_GEN_MINB) gen_kernel(const __grid
     __syncthreads();
     const uint64_t i0 = (lo - q_base) * 4, i1 = umin((hi - q_base) * 4, cur.s.n);
     gen_run<DT, DIST, SV_GEN_QPI>(ctx, cur.s, i0, i1, p.arena);
+    if (cur.fused) {  // uniform: the spec's exact-count edits inside this CTA's range
+      __syncthreads();
+      fused_edits<DT, DIST>(ctx, cur.s, cur.s.elem_offset + i0, cur.s.elem_offset + i1, p.arena);
+    }
   }
 }
 
@@ -188,12 +249,6 @@ static const void* gen_kernel_for(uint32_t dtype, uint32_t dist) {
 // pair for SWAP_PAIRS); the index of stratum s of [0, N) cut into k strata is
 // floor(s N / k) + mulhi64(x, len), x from INDEX block s.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ uint64_t stratum_index(const Ctx& c, uint32_t stream, uint64_t k, uint64_t st) {
-  const uint64_t start = (st * c.N) / k, end = ((st + 1) * c.N) / k;  // st < 2^21, N <= 2^40
-  const uint4 w = draw(c.rk, stream, P_INDEX, st);
-  const uint64_t x = ((uint64_t)w.x << 32) | w.y;
-  return start + __umul64hi(x, end - start);
-}
 
 template <int DT, int DIST>
 __device__ void fix_one(const Ctx& c, const syn_spec& s, uint64_t u, uint8_t* arena) {
@@ -218,21 +273,7 @@ __device__ void fix_one(const Ctx& c, const syn_spec& s, uint64_t u, uint8_t* ar
   }
   const uint64_t g = stratum_index(c, pc.stream, pc.count, u);
   if (g < lo || g >= hi) return;
-  const uint64_t v2 = value_at<DT, DIST>(c, g, 1);
-  uint64_t v3;
-  if constexpr (is_float(DT)) {
-    const float f = __double2float_rn(pc.value);
-    if (pc.kind == SV_PERT_COUNT_SET) {
-      v3 = from_f32<DT>(f);
-    } else {
-      const uint32_t b = (uint32_t)v2;
-      v3 = finite_bits<DT>(b) ? from_f32<DT>(__fadd_rn(to_f32<DT>(b), f)) : from_f32<DT>(f);
-    }
-  } else {
-    v3 = pc.kind == SV_PERT_COUNT_SET ? ((uint64_t)pc.ivalue & width_mask(DT))
-                                      : ((v2 + (uint64_t)pc.ivalue) & width_mask(DT));
-  }
-  put(g, v3);
+  put(g, count_edit_bits<DT, DIST>(c, pc, g));
 }
 
 __device__ void fix_dispatch(const Ctx& c, const syn_spec& s, uint64_t u, uint8_t* arena) {

@@ -37,6 +37,8 @@ struct DevSpec {
   syn_spec s;
   uint64_t work_begin;  // first unit inside its group's unit range
   uint64_t fix_begin;   // first thread in the exact-count fixup's list
+  uint32_t fused;       // exact-count edits applied by the generator CTAs (no fixup threads)
+  uint32_t pad;
 };
 
 // compare table entry: the caller's pair plus scheduling data
@@ -88,10 +90,19 @@ SV_HD inline uint64_t gen_tiles(const syn_spec& s) {
 SV_HD inline uint64_t gen_units(const syn_spec& s) {
   return s.dist == SV_DOTLIKE ? 0 : kGenEntryUnits + (s.n + 3) / 4;
 }
+// exact-count edits a generator CTA applies itself, at most, per entry it
+// touches (more strata than this in a CTA's slice: the fixup kernel does them)
+constexpr int kMaxFusedEdits = 64;
+
 SV_HD inline uint64_t fix_units(const syn_spec& s) {
   if (s.cand_offset == SV_NO_OUTPUT) return 0;
   const uint32_t k = s.pcount.kind;
   return (k == SV_PERT_COUNT_SET || k == SV_PERT_COUNT_ADD || k == SV_PERT_SWAP_PAIRS) ? s.pcount.count : 0;
+}
+
+// strata the exact-count edits cut [0, N) into (two per swapped pair)
+SV_HD inline uint64_t fix_strata(const syn_spec& s) {
+  return s.pcount.kind == SV_PERT_SWAP_PAIRS ? 2 * s.pcount.count : s.pcount.count;
 }
 
 // ---- generator ----

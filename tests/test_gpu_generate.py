@@ -172,6 +172,38 @@ def test_chunks_equal_whole_on_gpu(dev):
     assert np.array_equal(a.cpu().numpy(), h)
 
 
+@pytest.mark.parametrize("case", [
+    # few strata per CTA: the generating CTAs apply the edits (up to ~20 in one CTA here)
+    dict(dtype="f32", dist="uniform", n=1 << 20, p0=-1.0, p1=1.0, pcount=W.Perturb("count_set", stream=2, count=2000,
+                                                                              value=float("inf"))),
+    dict(dtype="i64", dist="permutation", n=1 << 20, pcount=W.Perturb("swap_pairs", stream=2, count=700)),
+    dict(dtype="f16", dist="uniform", n=300001, p0=-4.0, p1=4.0, pcount=W.Perturb("count_add", stream=2, count=90,
+                                                                               value=0.125)),
+    dict(dtype="bf16", dist="raw_bits", n=77777, pcount=W.Perturb("swap_pairs", stream=2, count=11)),
+    # dense strata: the fixup kernel applies them
+    dict(dtype="f32", dist="uniform", n=1000, p0=-1.0, p1=1.0, pcount=W.Perturb("count_set", stream=2, count=500,
+                                                                             value=-3.0)),
+    dict(dtype="i64", dist="permutation", n=4096, pcount=W.Perturb("swap_pairs", stream=2, count=1000)),
+    dict(dtype="bf16", dist="normal", n=20000, p0=0.0, p1=1.0, pcount=W.Perturb("count_add", stream=2, count=300,
+                                                                              value=0.5)),
+    dict(dtype="i32", dist="int_range", n=5000, i0=-9, i1=9, pcount=W.Perturb("count_add", stream=2, count=5000,
+                                                                            ivalue=1)),
+])
+def test_exact_count_edits_sparse_and_dense(dev, case):
+    kw = dict(case)
+    n = kw.pop("n")
+    sz = W.DTYPE_BYTES[kw["dtype"]]
+    spec = W.GenSpec(n=n, seed=11, stream=4, ref_offset=0, cand_offset=(n * sz + 255) // 256 * 256, **kw)
+    g, h = gen_both(dev, [[spec]], 2 * spec.cand_offset)
+    check_spec_outputs(g, h, spec)
+    ref = _view(g, 0, spec.dtype, n)
+    cand = _view(g, spec.cand_offset, spec.dtype, n)
+    if spec.pcount.kind == "swap_pairs":
+        assert np.count_nonzero(ref != cand) <= 2 * spec.pcount.count
+    else:
+        assert np.count_nonzero(ref != cand) <= spec.pcount.count
+
+
 @pytest.mark.parametrize("n_specs", [1, 8, 9, 40])
 def test_many_specs_one_call(dev, n_specs):
     # inline (<= 8) and uploaded tables, mixed kinds grouped per launch
