@@ -1,6 +1,8 @@
 // abi.cu -- the C ABI of synverify.h: host-side validation, workspace
 // layout, table upload and kernel launches.  No device memory is allocated
-// here; every device buffer comes from the caller.
+// here; every device buffer comes from the caller.  Entry tables larger than
+// the launch parameters go up from pinned host staging buffers that the
+// library allocates on first need and reuses for the life of the process.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -176,17 +178,113 @@ struct Group {
   LaunchShape sh;
 };
 
+// stable grouping by a small key (< kMaxKey; validated dtypes and
+// distributions): a counting sort, linear in n
+constexpr uint32_t kMaxKey = 64;
 template <class KeyFn>
 static void group_by(int n, KeyFn key, std::vector<int>& order, std::vector<Group>& groups) {
-  order.resize(n);
-  for (int i = 0; i < n; ++i) order[i] = i;
-  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return key(a) < key(b); });
+  uint32_t count[kMaxKey] = {0}, start[kMaxKey];
+  for (int i = 0; i < n; ++i) ++count[key(i) % kMaxKey];
   groups.clear();
-  for (int k = 0; k < n; ++k) {
-    if (groups.empty() || groups.back().key != key(order[k])) groups.push_back(Group{key(order[k]), k, k, 0, 0, {0, 1}});
-    groups.back().end = k + 1;
+  uint32_t at = 0;
+  for (uint32_t k = 0; k < kMaxKey; ++k) {
+    start[k] = at;
+    if (count[k]) groups.push_back(Group{k, (int)at, (int)(at + count[k]), 0, 0, {0, 1}});
+    at += count[k];
   }
+  order.resize(n);
+  for (int i = 0; i < n; ++i) order[start[key(i) % kMaxKey]++] = i;
 }
+
+// ---------------------------------------------------------------------------
+// pinned host staging for entry tables: a buffer is reused once the copy last
+// issued from it has completed (an event recorded after that copy); tables
+// beyond kMaxStaging, or when pinned memory is unavailable, go up from
+// ordinary host memory instead
+// ---------------------------------------------------------------------------
+namespace {
+constexpr size_t kMaxStaging = size_t(16) << 20;
+constexpr size_t kMaxStagingBuffers = 64;
+struct StagingBuf {
+  int dev;
+  void* host;
+  size_t cap;
+  cudaEvent_t done;
+  bool claimed;
+};
+std::mutex g_stage_mu;
+std::vector<StagingBuf*> g_stage;  // kept for the life of the process
+
+bool copy_finished(cudaEvent_t e) {
+  const cudaError_t q = cudaEventQuery(e);
+  if (q == cudaErrorNotReady && cudaPeekAtLastError() == cudaErrorNotReady) cudaGetLastError();
+  return q == cudaSuccess;
+}
+
+StagingBuf* claim_staging(size_t bytes) {
+  int dev = 0;
+  if (bytes == 0 || bytes > kMaxStaging || cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  std::lock_guard<std::mutex> lk(g_stage_mu);
+  for (StagingBuf* b : g_stage)
+    if (b->dev == dev && !b->claimed && b->cap >= bytes && copy_finished(b->done)) {
+      b->claimed = true;
+      return b;
+    }
+  if (g_stage.size() >= kMaxStagingBuffers) return nullptr;
+  size_t cap = size_t(64) << 10;
+  while (cap < bytes) cap *= 2;
+  void* h = nullptr;
+  if (cudaHostAlloc(&h, cap, cudaHostAllocPortable) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  cudaEvent_t e;
+  if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFreeHost(h);
+    return nullptr;
+  }
+  StagingBuf* b = new StagingBuf{dev, h, cap, e, true};
+  g_stage.push_back(b);
+  return b;
+}
+
+// a host table of n entries of T: pinned when it will be uploaded and fits a
+// staging buffer, else ordinary memory; upload() copies it to the device and
+// marks the buffer busy until that copy completes
+template <class T>
+class HostTable {
+ public:
+  HostTable(int n, bool upload) : n_(n) {
+    if (upload) buf_ = claim_staging(sizeof(T) * (size_t)n);
+    if (buf_) {
+      p_ = static_cast<T*>(buf_->host);
+    } else {
+      vec_.resize(n);
+      p_ = vec_.data();
+    }
+  }
+  ~HostTable() {  // the host copy is read until the call returns
+    if (buf_) {
+      std::lock_guard<std::mutex> lk(g_stage_mu);
+      buf_->claimed = false;
+    }
+  }
+  T* data() { return p_; }
+  T& operator[](int i) { return p_[i]; }
+  cudaError_t upload(void* dst, cudaStream_t st) {
+    const cudaError_t e = cudaMemcpyAsync(dst, p_, sizeof(T) * (size_t)n_, cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess || !buf_) return e;
+    return cudaEventRecord(buf_->done, st);
+  }
+
+ private:
+  int n_;
+  StagingBuf* buf_ = nullptr;
+  T* p_ = nullptr;
+  std::vector<T> vec_;
+};
+}  // namespace
 
 static size_t spec_table_bytes(int n) { return n > SV_INLINE_ENTRIES ? align_up(sizeof(DevSpec) * (size_t)n) : 0; }
 static size_t pair_table_bytes(int n) { return n > SV_INLINE_ENTRIES ? align_up(sizeof(DevPair) * (size_t)n) : 0; }
@@ -299,7 +397,7 @@ int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena
   std::vector<int> order;
   std::vector<Group> groups;
   group_by(n_specs, [&](int i) { return specs[i].dtype * 8u + specs[i].dist; }, order, groups);
-  std::vector<DevSpec> tab(n_specs);
+  HostTable<DevSpec> tab(n_specs, need != 0);
   for (Group& g : groups) {
     for (int k = g.begin; k < g.end; ++k) {
       const syn_spec& s = specs[order[k]];
@@ -332,8 +430,7 @@ int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena
   }
   const DevSpec* dev = nullptr;
   if (need) {
-    if (cudaMemcpyAsync(d_ws, tab.data(), sizeof(DevSpec) * tab.size(), cudaMemcpyHostToDevice, st) != cudaSuccess)
-      return SV_ECUDA;
+    if (tab.upload(d_ws, st) != cudaSuccess) return SV_ECUDA;
     dev = static_cast<const DevSpec*>(d_ws);
   }
   uint8_t* arena = static_cast<uint8_t*>(d_arena);
@@ -362,7 +459,7 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
   std::vector<int> order;
   std::vector<Group> groups;
   group_by(n_pairs, [&](int i) { return pairs[i].dtype; }, order, groups);
-  std::vector<DevPair> tab(n_pairs);
+  HostTable<DevPair> tab(n_pairs, tb != 0);
   uint64_t slot_base = 0;
   for (Group& g : groups) {
     for (int k = g.begin; k < g.end; ++k) {
@@ -386,8 +483,7 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
   uint8_t* ws = static_cast<uint8_t*>(d_ws);
   const DevPair* dev = nullptr;
   if (tb) {
-    if (cudaMemcpyAsync(ws, tab.data(), sizeof(DevPair) * tab.size(), cudaMemcpyHostToDevice, st) != cudaSuccess)
-      return SV_ECUDA;
+    if (tab.upload(ws, st) != cudaSuccess) return SV_ECUDA;
     dev = reinterpret_cast<const DevPair*>(ws);
   }
   Partial* partials = reinterpret_cast<Partial*>(ws + tb);

@@ -29,8 +29,14 @@ constexpr int kStagedStarts = 2048;        // tables up to this size are searche
 // (staging it, building its context, flushing its statistics) plus its
 // elements, and each CTA of a persistent grid takes an equal contiguous slice
 // of the units, so many small entries spread as evenly as a few large ones.
-constexpr uint64_t kGenEntryUnits = 1024;  // generator: units are 4-element quanta
-constexpr uint64_t kCmpEntryUnits = 512;   // compare: units are 16-byte vectors
+#ifndef SV_GEN_ENTRY_UNITS
+#define SV_GEN_ENTRY_UNITS 2048
+#endif
+#ifndef SV_CMP_ENTRY_UNITS
+#define SV_CMP_ENTRY_UNITS 2048
+#endif
+constexpr uint64_t kGenEntryUnits = SV_GEN_ENTRY_UNITS;  // generator: units are 4-element quanta
+constexpr uint64_t kCmpEntryUnits = SV_CMP_ENTRY_UNITS;  // compare: units are 16-byte vectors
 
 // generator table entry: the caller's spec plus scheduling data
 struct DevSpec {
