@@ -374,7 +374,7 @@ def ours_arm(args, rank, world):
                     "peak_kind": "%s (%s)" % (peak_kind, "hbm_gbs"), "traffic": traffic}
     line = {
         "metric": METRIC,
-        "value": world * step_bytes / (total_ms * 1e-3 / args.steps) / 1e9,
+        "value": job_throughput(step_bytes, args.steps, world, total_ms * 1e-3),
         "unit": "GB/s",
         "n_gpus": world,
         "steps": args.steps,
@@ -397,7 +397,7 @@ def ours_arm(args, rank, world):
         "gen_ms": gen_ms,
         "verify_ms": ver_ms,
         "roofline": roofline,
-        "e2e": {"value": world * step_bytes * e2e_steps / e2e_s / 1e9, "unit": "GB/s",
+        "e2e": {"value": job_throughput(step_bytes, e2e_steps, world, e2e_s), "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps},
         "clocks": clocks,
         "gpu_launches": launches_per_step * args.steps,
@@ -429,13 +429,22 @@ def barrier(world):
 
 
 def max_over_ranks(x, world):
+    """The largest of the ranks' x (the slowest rank's time): one all-reduce on
+    the process group's device (CUDA for NCCL, host memory for gloo)."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_throughput(bytes_per_rank_step, steps, world, slowest_s):
+    """Whole-job GB/s of N independent replicas: every rank processes the same
+    bytes per step, and the job takes as long as its slowest rank."""
+    return world * bytes_per_rank_step * steps / slowest_s / 1e9
 
 
 def main():
