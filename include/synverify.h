@@ -11,15 +11,18 @@
  * - Plain C types only.  Device buffers are raw device pointers with a byte
  *   size; spec/pair tables are HOST arrays, read during the call only.
  * - Ownership: the caller owns every buffer.  The library allocates no device
- *   or pinned memory and keeps no state between calls (apart from a per-device
- *   cache of the SM count and occupancy, filled on first use).
+ *   memory.  It keeps two kinds of state between calls: a per-device cache of
+ *   the SM count and occupancy, and pinned host staging buffers for entry
+ *   tables (allocated on first need, at most 64 buffers of at most 16 MiB,
+ *   kept for the life of the process).
  * - Execution: every call enqueues work on `stream` and returns without
  *   waiting; results are written to device memory.  Calls on different streams
  *   are independent when their workspaces and outputs do not overlap.  A table
- *   larger than SV_INLINE_ENTRIES entries is copied to the workspace with
- *   cudaMemcpyAsync from the caller's host array; from pageable memory the
- *   driver may wait for the stream before that copy (pass pinned memory to
- *   keep such a call fully asynchronous).
+ *   larger than SV_INLINE_ENTRIES entries is built in a pinned staging buffer
+ *   and copied to the workspace with cudaMemcpyAsync; a staging buffer is
+ *   reused only after the copy issued from it has completed.  (If no staging
+ *   buffer can be had, the table goes from ordinary host memory, and the
+ *   driver may then wait for the stream before that copy.)
  * - Errors: 0 on success, a negative SV_E* status otherwise.  All arguments are
  *   validated on the host before anything is enqueued, so a validation error
  *   leaves device memory untouched.  SV_ECUDA reports a CUDA launch or copy
