@@ -162,8 +162,8 @@ def run_round(task: Task, candidate_src: str, reference_src: str, work_dir: str,
         return RoundResult(1, 0, 0.0, reward(1, 0, 0.0), None, first_failed, stages, cand.log)
 
     # P of Eq. 3 on the largest stage: mean latency of `runs` launches (CUDA
-    # events on the launching stream, after warm-up); the operation is applied
-    # to a scratch copy so the validated output stays as it was
+    # events on the launching stream, after warm-up), reusing the candidate's
+    # output buffer of that stage now that its verdict is in
     n = task.stages[-1]
     a_off, b_off, _, c_off = layout[-1]
     for _ in range(3):
