@@ -505,7 +505,10 @@ int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, 
   if (n_stages > 0 && (!d_results || (cand_bytes && !d_cand) || (ref_bytes && !d_ref))) return SV_EINVAL;
   if (!ws_ok(d_ws, ws_bytes, sv_progressive_workspace_bytes(stages, n_stages))) return SV_EWORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(d_first_failed, 0xFF, sizeof(int32_t), st) != cudaSuccess) return SV_ECUDA;
+  // the first group's combine sets the flag (failing stage or -1); an empty
+  // ladder only clears it
+  if (n_stages == 0) return cudaMemsetAsync(d_first_failed, 0xFF, sizeof(int32_t), st) == cudaSuccess ? SV_OK
+                                                                                                        : SV_ECUDA;
   Partial* partials = static_cast<Partial*>(d_ws);
   const uint8_t* cand = static_cast<const uint8_t*>(d_cand);
   const uint8_t* ref = static_cast<const uint8_t*>(d_ref);
@@ -531,10 +534,12 @@ int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, 
       tab[k].pad = 0;
       u += cmp_units(tab[k].p);
     }
-    // the compare returns at once when an earlier group failed; the combine
-    // then reports the group as skipped
-    cudaError_t e = launch_compare_group(dtype, tab, nullptr, ng, units, sh, cand, ref, partials, d_first_failed, st);
-    if (e == cudaSuccess) e = launch_combine(tab, nullptr, ng, partials, d_results, d_first_failed, 0, st);
+    // the compare of a later group returns at once when an earlier group
+    // failed; the combine then reports the group as skipped
+    const bool first = g.first == 0;
+    cudaError_t e = launch_compare_group(dtype, tab, nullptr, ng, units, sh, cand, ref, partials,
+                                         first ? nullptr : d_first_failed, st);
+    if (e == cudaSuccess) e = launch_combine(tab, nullptr, ng, partials, d_results, d_first_failed, first, st);
     if (e != cudaSuccess) return SV_ECUDA;
   }
   return SV_OK;

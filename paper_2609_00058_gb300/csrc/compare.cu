@@ -43,7 +43,7 @@ struct CombParams {
   const Partial* partials;
   vc_result* results;
   int32_t* flag;
-  int stage;
+  int first_group;  // progressive: the ladder's first group (the flag is not yet set)
 };
 
 template <class P>
@@ -477,7 +477,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant
 __global__ void __launch_bounds__(kThreads) combine_stages_kernel(const __grid_constant__ CombParams p) {
   __shared__ vc_result res[SV_INLINE_ENTRIES];
   const int e = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (*p.flag >= 0) {  // an earlier group failed: nothing of this group ran
+  if (!p.first_group && *p.flag >= 0) {  // an earlier group failed: nothing of this group ran
     if (threadIdx.x < p.n) p.results[pentry(p, threadIdx.x)->orig] = skipped_result();
     return;
   }
@@ -497,7 +497,7 @@ __global__ void __launch_bounds__(kThreads) combine_stages_kernel(const __grid_c
       p.results[dp->orig] = res[i];
       if (!res[i].pass) failed = (int)dp->orig;
     }
-    if (failed >= 0) *p.flag = failed;
+    if (failed >= 0 || p.first_group) *p.flag = failed;  // the first group also clears it
   }
 }
 
@@ -551,14 +551,14 @@ cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevP
 }
 
 cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const Partial* partials,
-                           vc_result* results, int32_t* flag, int stage, cudaStream_t st) {
+                           vc_result* results, int32_t* flag, int first_group, cudaStream_t st) {
   if (n == 0) return cudaSuccess;
   CombParams cp;
   fill_pairs(cp, host, dev, n);
   cp.partials = partials;
   cp.results = results;
   cp.flag = flag;
-  cp.stage = stage;
+  cp.first_group = first_group;
   if (flag) {  // a progressive group: one CTA, stages in order
     if (n > SV_INLINE_ENTRIES || dev) return cudaErrorInvalidValue;
     combine_stages_kernel<<<1, kThreads, 0, st>>>(cp);

@@ -126,6 +126,6 @@ cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevP
                                  LaunchShape sh, const uint8_t* cand, const uint8_t* ref, Partial* partials,
                                  const int32_t* flag, cudaStream_t st);
 cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const Partial* partials,
-                           vc_result* results, int32_t* flag, int stage, cudaStream_t st);
+                           vc_result* results, int32_t* flag, int first_group, cudaStream_t st);
 
 }  // namespace sv
