@@ -204,6 +204,30 @@ def test_exact_count_edits_sparse_and_dense(dev, case):
         assert np.count_nonzero(ref != cand) <= spec.pcount.count
 
 
+@pytest.mark.parametrize("kw", [
+    dict(dtype="f32", dist="uniform", p0=-3.0, p1=7.0, specials=("nan", "dup", "denorm"), special_rate=0.01,
+         pelem=W.Perturb("rate_add_pm", stream=5, rate=0.01, value=0.5)),
+    dict(dtype="bf16", dist="normal", p0=5.0, p1=10.0, pelem=W.Perturb("rel_noise", stream=6, value=2.0 ** -9)),
+    dict(dtype="i64", dist="permutation", specials=("dup", "imin"), special_rate=0.01,
+         pcount=W.Perturb("swap_pairs", stream=7, count=3)),
+    dict(dtype="i64", dist="int_range", i0=-(2 ** 40), i1=2 ** 40, pcount=W.Perturb("count_add", stream=8, count=5,
+                                                                                  ivalue=-1)),
+    dict(dtype="u32", dist="raw_bits", pcount=W.Perturb("count_set", stream=9, count=2, ivalue=7)),
+])
+def test_chunk_at_the_top_of_the_largest_logical_range(dev, kw):
+    # a chunk ending at logical index 2^40: 64-bit counters, permutation
+    # constants beyond 32 bits and strata of about 2^38 elements
+    ln = 1 << 40
+    n = 20001
+    eo = ln - n - 3  # the quantum-aligned start (multiple of 4) of a ragged chunk
+    eo -= eo % 4
+    sz = W.DTYPE_BYTES[kw["dtype"]]
+    spec = W.GenSpec(n=n, seed=77, stream=1, ref_offset=0, cand_offset=(n * sz + 255) // 256 * 256,
+                     elem_offset=eo, logical_n=ln, **kw)
+    g, h = gen_both(dev, [[spec]], 2 * spec.cand_offset)
+    check_spec_outputs(g, h, spec)
+
+
 @pytest.mark.parametrize("n_specs", [1, 8, 9, 40])
 def test_many_specs_one_call(dev, n_specs):
     # inline (<= 8) and uploaded tables, mixed kinds grouped per launch
