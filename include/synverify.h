@@ -268,6 +268,12 @@ int verify_compare_noalloc(const vc_pair* pairs, int n_pairs, const void* d_cand
 const char* sv_strerror(int status);
 int sv_abi_version(void);
 
+/* Instrumentation (no counterpart in the paper): the number of CUDA kernels
+ * this library has launched in this process, on all devices and streams,
+ * since it was loaded.  Read it before and after a piece of work to count that
+ * work's launches.  Thread-safe; never fails. */
+uint64_t sv_kernel_launches(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -134,6 +134,7 @@ EXPORTS = [
     ("verify_compare_noalloc", C.c_int, [C.POINTER(vc_pair), C.c_int, _VP, _SZ, _VP, _SZ, _VP, _VP]),
     ("sv_strerror", C.c_char_p, [C.c_int]),
     ("sv_abi_version", C.c_int, []),
+    ("sv_kernel_launches", C.c_uint64, []),
 ]
 
 _lib = None

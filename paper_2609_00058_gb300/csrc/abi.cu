@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <mutex>
 #include <vector>
@@ -39,6 +40,11 @@ struct CapEntry {
 std::mutex g_mu;
 std::vector<CapEntry> g_caps;
 }  // namespace
+
+namespace {
+std::atomic<uint64_t> g_launches{0};
+}
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 uint32_t grid_cap_for(const void* fn, size_t dyn_smem) {
   int dev = 0;
@@ -318,6 +324,8 @@ using namespace sv;
 extern "C" {
 
 int sv_abi_version(void) { return SV_ABI_VERSION; }
+
+uint64_t sv_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
 
 const char* sv_strerror(int status) {
   switch (status) {

@@ -547,6 +547,7 @@ cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevP
     case SV_I64: cmp_kernel<SV_I64><<<sh.grid, kThreads, 0, st>>>(cp); break;
     default: cmp_kernel<SV_U32><<<sh.grid, kThreads, 0, st>>>(cp); break;
   }
+  count_launch();
   return cudaGetLastError();
 }
 
@@ -566,6 +567,7 @@ cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const
     const uint64_t blocks = ((uint64_t)n * 32 + kThreads - 1) / kThreads;
     combine_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(cp);
   }
+  count_launch();
   return cudaGetLastError();
 }
 

@@ -529,6 +529,7 @@ cudaError_t launch_generate_group(uint32_t dtype, uint32_t dist, const DevSpec* 
 #undef SV_CASE
     default: return cudaErrorInvalidValue;
   }
+  count_launch();
   return cudaGetLastError();
 }
 
@@ -542,6 +543,7 @@ cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_
   gp.arena = arena;
   const uint64_t blocks = (total_units + kThreads - 1) / kThreads;
   fixup_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(gp);
+  count_launch();
   return cudaGetLastError();
 }
 
@@ -551,6 +553,7 @@ static cudaError_t launch_dot(const DotParams& dp, uint64_t tiles, cudaStream_t 
   const uint32_t cap = grid_cap_for(fn, kDotSmem);
   const unsigned grid = (unsigned)std::min<uint64_t>(tiles, cap);
   dot_kernel<DT, A16><<<grid, kThreads, kDotSmem, st>>>(dp);
+  count_launch();
   return cudaGetLastError();
 }
 

@@ -74,3 +74,25 @@ def test_empty_ladder_and_empty_stage(dev):
     res, ff = sv.progressive([W.Pair("f32", 0, 0, 0)], a, a)
     g = sv.decode_results(res, 1)[0]
     assert int(ff.item()) == -1 and g["pass"] == 1 and g["state"] == 1 and g["first_mismatch"] == -1
+
+
+def test_library_counts_its_own_launches(dev):
+    # one generator launch for a one-kind batch (its sparse exact-count edit is
+    # applied in the generating CTAs), then one compare and one ordered
+    # combine per stage group of the ladder (five small fp32 stages: one group)
+    import torch
+    wl = W.progressive_ladder((10, 12, 14, 16, 18), deviate_stage=2, special_rate=1e-3)
+    a = torch.zeros(wl.arena_bytes, dtype=torch.uint8, device=dev)
+    lib = sv.lib()
+    n0 = lib.sv_kernel_launches()
+    sv.generate(wl.gen_calls[0], a)
+    n1 = lib.sv_kernel_launches()
+    res, ff = sv.progressive(wl.pairs, a, a)
+    n2 = lib.sv_kernel_launches()
+    assert (n1 - n0, n2 - n1) == (1, 2)
+    assert int(ff.item()) == 2
+    # two pairs of different dtypes: a compare per dtype and one combine
+    pairs = [W.Pair("f32", 1000, 0, 0), W.Pair("i32", 1000, 4096, 4096)]
+    n3 = lib.sv_kernel_launches()
+    sv.compare(pairs, a, a)
+    assert lib.sv_kernel_launches() - n3 == 3
