@@ -264,6 +264,20 @@ int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, 
 int verify_compare_noalloc(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t cand_bytes,
                            const void* d_ref, size_t ref_bytes, vc_result* d_results, sv_stream_t stream);
 
+/* The Box-Muller step of the normal distribution (Sec. 4.2.1: normal test
+ * values over broad ranges) on caller-supplied 32-bit words: pair i,
+ * (d_words[2i], d_words[2i+1]) = (wa, wb), gives
+ *   d_z[2i]   = r cos(theta),  d_z[2i+1] = r sin(theta),
+ *   r = sqrt(-2 ln u1), u1 = ((wa >> 8) + 1) 2^-24,  theta = 2 pi (wb >> 8) 2^-24,
+ * in fp32, exactly the values syn_generate makes for N(0, 1) from the same
+ * VALUE words (so the transform can be checked alone, on any words).
+ * Within 4 ulp of the transform computed in fp64 and rounded once.
+ * d_words: n_pairs x 2 uint32 on the device; d_z: n_pairs x 2 float on the
+ * device; both 8-byte aligned (SV_EALIGN) and caller-owned.  n_pairs = 0 is a
+ * no-op; n_pairs > SV_MAX_LOGICAL_N / 2: SV_ERANGE; null pointers: SV_EINVAL.
+ * Asynchronous on `stream`; allocates nothing. */
+int syn_box_muller(const uint32_t* d_words, size_t n_pairs, float* d_z, sv_stream_t stream);
+
 /* Static description of a status code. */
 const char* sv_strerror(int status);
 int sv_abi_version(void);

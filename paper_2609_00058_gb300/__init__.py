@@ -135,6 +135,7 @@ EXPORTS = [
     ("sv_strerror", C.c_char_p, [C.c_int]),
     ("sv_abi_version", C.c_int, []),
     ("sv_kernel_launches", C.c_uint64, []),
+    ("syn_box_muller", C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
 ]
 
 _lib = None
@@ -292,6 +293,17 @@ def progressive(stages, cand, ref, results=None, first_failed=None, workspace=No
                                   _stream_ptr(stream))
     _ok(rc, "verify_progressive")
     return results, first_failed
+
+
+def box_muller(words, out=None, stream=None):
+    """syn_box_muller: the generator's Box-Muller step on a CUDA uint32 tensor
+    of word pairs; returns (or fills) a float32 tensor of the same length."""
+    import torch
+    n_pairs = words.numel() // 2
+    if out is None:
+        out = torch.empty(2 * n_pairs, dtype=torch.float32, device=words.device)
+    _ok(lib().syn_box_muller(words.data_ptr(), n_pairs, out.data_ptr(), _stream_ptr(stream)), "syn_box_muller")
+    return out
 
 
 def decode_results(results, n: int) -> List[dict]:

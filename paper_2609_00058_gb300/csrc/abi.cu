@@ -327,6 +327,14 @@ int sv_abi_version(void) { return SV_ABI_VERSION; }
 
 uint64_t sv_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
 
+int syn_box_muller(const uint32_t* d_words, size_t n_pairs, float* d_z, sv_stream_t stream) {
+  if (n_pairs == 0) return SV_OK;
+  if (!d_words || !d_z) return SV_EINVAL;
+  if (n_pairs > SV_MAX_LOGICAL_N / 2) return SV_ERANGE;
+  if ((reinterpret_cast<uintptr_t>(d_words) | reinterpret_cast<uintptr_t>(d_z)) & 7) return SV_EALIGN;
+  return status_of(launch_box_muller(d_words, n_pairs, d_z, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 const char* sv_strerror(int status) {
   switch (status) {
     case SV_OK: return "ok";

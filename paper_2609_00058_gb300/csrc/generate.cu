@@ -500,6 +500,19 @@ __global__ void __launch_bounds__(kThreads, SV_DOT_MINB) dot_kernel(const __grid
 }
 
 // ---------------------------------------------------------------------------
+// the Box-Muller step alone, on caller words (syn_box_muller): pair i of
+// words gives the two normals the generator makes from the same words
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) box_muller_kernel(const uint2* w, uint64_t n_pairs, float2* z) {
+  for (uint64_t i = (uint64_t)blockIdx.x * kThreads + threadIdx.x; i < n_pairs; i += (uint64_t)gridDim.x * kThreads) {
+    const uint2 p = w[i];
+    float z0, z1;
+    box_muller(p.x, p.y, z0, z1);
+    z[i] = make_float2(z0, z1);
+  }
+}
+
+// ---------------------------------------------------------------------------
 // host launchers
 // ---------------------------------------------------------------------------
 static void fill_params(GenParams& gp, const DevSpec* host, const DevSpec* dev, int n) {
@@ -553,6 +566,16 @@ static cudaError_t launch_dot(const DotParams& dp, uint64_t tiles, cudaStream_t 
   const uint32_t cap = grid_cap_for(fn, kDotSmem);
   const unsigned grid = (unsigned)std::min<uint64_t>(tiles, cap);
   dot_kernel<DT, A16><<<grid, kThreads, kDotSmem, st>>>(dp);
+  count_launch();
+  return cudaGetLastError();
+}
+
+cudaError_t launch_box_muller(const uint32_t* words, uint64_t n_pairs, float* z, cudaStream_t st) {
+  if (n_pairs == 0) return cudaSuccess;
+  const void* fn = reinterpret_cast<const void*>(box_muller_kernel);
+  const uint64_t blocks = std::min<uint64_t>((n_pairs + kThreads - 1) / kThreads, grid_cap_for(fn));
+  box_muller_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(reinterpret_cast<const uint2*>(words), n_pairs,
+                                                            reinterpret_cast<float2*>(z));
   count_launch();
   return cudaGetLastError();
 }

@@ -121,6 +121,7 @@ cudaError_t launch_generate_group(uint32_t dtype, uint32_t dist, const DevSpec* 
 cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_t units, uint8_t* arena,
                          cudaStream_t st);
 cudaError_t launch_dotlike(const DevSpec& spec, uint8_t* arena, cudaStream_t st);
+cudaError_t launch_box_muller(const uint32_t* words, uint64_t n_pairs, float* z, cudaStream_t st);
 
 // ---- compare ----
 LaunchShape compare_shape(uint32_t dtype, uint64_t units, uint64_t tiles);

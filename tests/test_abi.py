@@ -180,3 +180,12 @@ def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(sv, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="not built"):
         sv.lib()
+
+
+def test_box_muller_entry_validates_before_any_launch():
+    lib = sv.lib()
+    assert lib.syn_box_muller(None, 0, None, None) == 0            # no-op
+    assert lib.syn_box_muller(None, 4, 0x1000, None) == -1         # null words
+    assert lib.syn_box_muller(0x1004, 4, 0x2000, None) == -2       # 4-byte aligned words
+    assert lib.syn_box_muller(0x1000, 4, 0x2004, None) == -2       # 4-byte aligned output
+    assert lib.syn_box_muller(0x1000, (1 << 39) + 1, 0x2000, None) == -3

@@ -1,0 +1,85 @@
+"""The generator's fp32 Box-Muller step (normal values, Sec. 4.2.1) through
+syn_box_muller, against the oracle's fp64 transform rounded once.
+
+Both inputs of the transform are 24-bit integers (wa >> 8 and wb >> 8), so
+each factor is checked on its whole domain: every radius (angle 0, where
+z0 = r exactly and z1 = 0) and every angle at several radii; then random
+pairs.  The bound is the benchmark spec's 4 ulp (ordered-integer distance); the
+tests also require most values to be exact, and that syn_box_muller gives
+the generator's own N(0, 1) values on the generator's words.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2609_00058_gb300 as sv
+import workloads as W
+from gpu_util import device, ordered_f32
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    return device()
+
+
+def gpu_bm(words, dev):
+    import torch
+    w = torch.from_numpy(words.view(np.int32)).to(dev)
+    return sv.box_muller(w).cpu().numpy()
+
+
+def ulp_dist(a, b):
+    return np.abs(ordered_f32(a.view(np.uint32)) - ordered_f32(b.view(np.uint32)))
+
+
+def test_every_radius(dev):
+    k = np.arange(1 << 24, dtype=np.uint32)
+    rng = np.random.default_rng(1)
+    words = np.empty(2 * k.size, np.uint32)
+    words[0::2] = (k << 8) | rng.integers(0, 256, k.size, dtype=np.uint32)  # low bits are ignored
+    words[1::2] = rng.integers(0, 256, k.size, dtype=np.uint32)             # angle 0
+    got, want = gpu_bm(words, dev), oracle.box_muller(words)
+    d = ulp_dist(got, want)
+    assert d.max() <= 2, d.max()
+    assert (d == 0).mean() > 0.6
+    assert np.array_equal(np.signbit(got[1::2]), np.signbit(want[1::2]))
+
+
+@pytest.mark.parametrize("a", [0, 1, 0x4DA7F6, 0xB2F0C3, 0xFFFFFE, 0xFFFFFF])
+def test_every_angle(dev, a):
+    k = np.arange(1 << 24, dtype=np.uint32)
+    words = np.empty(2 * k.size, np.uint32)
+    words[0::2] = np.uint32(a << 8)
+    words[1::2] = k << 8
+    got, want = gpu_bm(words, dev), oracle.box_muller(words)
+    d = ulp_dist(got, want)
+    assert d.max() <= 4, (a, d.max(), int(np.argmax(d)))
+    assert (d == 0).mean() > 0.5
+    # exact zeros of the quarter rotations keep their signs
+    z = want == 0
+    assert np.array_equal(got[z].view(np.uint32), want[z].view(np.uint32))
+
+
+def test_random_pairs(dev):
+    rng = np.random.default_rng(2)
+    words = rng.integers(0, 1 << 32, 2 * (1 << 23), dtype=np.uint64).astype(np.uint32)
+    got, want = gpu_bm(words, dev), oracle.box_muller(words)
+    d = ulp_dist(got, want)
+    assert d.max() <= 4
+    assert (d == 0).mean() > 0.5
+    assert (d <= 1).mean() > 0.95
+
+
+def test_same_values_as_the_generator(dev):
+    import torch
+    n = 1 << 16
+    spec = W.GenSpec("f32", "normal", n, seed=321, stream=5, ref_offset=0, p0=0.0, p1=1.0)
+    a = torch.zeros(4 * n, dtype=torch.uint8, device=dev)
+    sv.generate([spec], a)
+    words = np.concatenate([oracle.draw(321, 5, "value", b) for b in range(n // 4)]).astype(np.uint32)
+    got = gpu_bm(words, dev)
+    gen = a.cpu().numpy().view(np.float32)
+    # the generator adds mu = 0 to sigma * z, which turns -0 into +0
+    assert np.array_equal(got, gen) and np.array_equal(got[got != 0].view(np.uint32), gen[gen != 0].view(np.uint32))
