@@ -60,15 +60,18 @@ def load_peaks():
 
 
 def alu_peaks():
-    """Philox blocks and Box-Muller pairs per SM per cycle, measured now on
-    this GPU by paper_2609_00058_gb300/probes/alu_peak.cu (built on demand)."""
+    """Philox blocks, Box-Muller pairs and fp32 FMAs per SM per cycle of the
+    library's own device code, measured now on this GPU by
+    paper_2609_00058_gb300/probes/alu_peak.cu (built on demand)."""
     import subprocess
     src = os.path.join(ROOT, "paper_2609_00058_gb300", "probes", "alu_peak.cu")
     exe = os.path.join(ROOT, "paper_2609_00058_gb300", "_build", "alu_peak")
     try:
-        if not os.path.exists(exe) or os.path.getmtime(exe) < os.path.getmtime(src):
+        deps = [src] + [os.path.join(ROOT, "paper_2609_00058_gb300", "csrc", f) for f in ("sv_device.cuh", "sv_kernels.h")]
+        if not os.path.exists(exe) or os.path.getmtime(exe) < max(os.path.getmtime(d) for d in deps):
             from paper_2609_00058_gb300 import build as b
-            subprocess.run([b.nvcc(), *b.ARCH, "-O3", "-o", exe, src], check=True, capture_output=True, timeout=300)
+            subprocess.run([b.nvcc(), *b.ARCH, "-O3", "-std=c++17", "--fmad=false", "-o", exe, src], check=True,
+                           capture_output=True, timeout=300)
         out = subprocess.run([exe], check=True, capture_output=True, text=True, timeout=120).stdout
         return json.loads(out.strip().splitlines()[-1])
     except Exception as e:  # the roofline falls back to HBM alone

@@ -1,45 +1,31 @@
-// alu_peak.cu -- measures the two ALU rates that bound the normal-value
-// generator on this GPU: Philox-4x32-10 blocks and Box-Muller pairs per SM
-// per cycle, each run alone at full occupancy with no memory traffic.  The
-// generator's ALU roofline for a quantum is the sum of its blocks' and
-// pairs' cycle costs.  Prints one JSON line.  Not part of the library.
+// alu_peak.cu -- measures the ALU rates that bound the generator on this GPU:
+// Philox-4x32-10 blocks (two interleaved under one key, as the generator
+// draws them), Box-Muller pairs (the generator's own fp32 transform) and fp32
+// fused multiply-adds (scalar and packed), each run alone at full occupancy
+// with no memory traffic, per SM per cycle at the maximum clock.  The
+// generator's ALU roofline for a quantum is the sum of its blocks', pairs'
+// and FMAs' cycle costs.  Prints one JSON line.  Not part of the library.
 #include <cuda_runtime.h>
 
 #include <cstdint>
 #include <cstdio>
 
+#include "../csrc/sv_device.cuh"
+
 namespace {
-constexpr uint32_t kM0 = 0xD2511F53u, kM1 = 0xCD9E8D57u, kW0 = 0x9E3779B9u, kW1 = 0xBB67AE85u;
 constexpr int kIter = 256;
 constexpr int kFmaIter = 4096;  // long enough (about 0.5 ms a launch) for a steady clock
 
-__device__ __forceinline__ uint4 block(uint4 c, uint32_t k0, uint32_t k1) {
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    const uint64_t p0 = (uint64_t)kM0 * c.x, p1 = (uint64_t)kM1 * c.z;
-    c = make_uint4((uint32_t)(p1 >> 32) ^ c.y ^ (k0 + r * kW0), (uint32_t)p1, (uint32_t)(p0 >> 32) ^ c.w ^ (k1 + r * kW1),
-                   (uint32_t)p0);
-  }
-  return c;
-}
-
 __global__ void philox_kernel(uint32_t* out, uint32_t k0, uint32_t k1) {
+  const sv::RoundKeys rk = sv::round_keys(sv::Key{k0, k1});
   uint32_t acc = 0;
   const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
   for (int i = 0; i < kIter; i += 2) {
-    const uint4 a = block(make_uint4(t, i, 7, 0), k0, k1), b = block(make_uint4(t, i + 1, 7, 0), k0, k1);
+    uint4 a = make_uint4(t, i, 7, 0), b = make_uint4(t, i + 1, 7, 0);
+    sv::philox2_rk(a, b, rk);
     acc ^= a.x ^ a.y ^ a.z ^ a.w ^ b.x ^ b.y ^ b.z ^ b.w;
   }
   if (acc == 0x12345678u) out[t] = acc;  // keeps the work live
-}
-
-__device__ __forceinline__ void pair(uint32_t wa, uint32_t wb, float& z0, float& z1) {
-  const float u1 = __fmul_rn(__uint2float_rn((wa >> 8) + 1u), 0x1p-24f);
-  const float r = sqrtf(__fmul_rn(-2.0f, logf(u1)));
-  float s, c;
-  sincospif(__fmul_rn(__uint2float_rn(wb >> 8), 0x1p-23f), &s, &c);
-  z0 = __fmul_rn(r, c);
-  z1 = __fmul_rn(r, s);
 }
 
 __global__ void box_muller_kernel(uint32_t* out) {
@@ -48,8 +34,8 @@ __global__ void box_muller_kernel(uint32_t* out) {
   const uint32_t wa = t * 2654435761u, wb = t * 40503u + 17u;
   for (int i = 0; i < kIter; i += 2) {
     float a0, a1, b0, b1;
-    pair(wa + i * 0x9E3779B9u, wb ^ (i * 0x85EBCA6Bu), a0, a1);
-    pair(wa ^ (i * 0xC2B2AE35u), wb + i * 0x27D4EB2Fu, b0, b1);
+    sv::box_muller(wa + i * 0x9E3779B9u, wb ^ (i * 0x85EBCA6Bu), a0, a1);
+    sv::box_muller(wa ^ (i * 0xC2B2AE35u), wb + i * 0x27D4EB2Fu, b0, b1);
     acc += a0 + a1 + b0 + b1;
   }
   if (acc == 12345.0f) out[t] = 1;
