@@ -119,6 +119,53 @@ def test_specials_rate_and_kinds(oracle):
     assert np.all(u[nan] == 0x7FC00000)
 
 
+@pytest.mark.parametrize("rate", [1e-4, 1.0 / 256, 0.01, 0.3, 1.0])
+def test_special_rate_is_binomial(oracle, rate):
+    # the count of selected elements is binomial(n, rate); rate 1 selects all
+    n = 1 << 18
+    s = W.GenSpec("f32", "uniform", n, seed=5, stream=3, ref_offset=0, p0=-1.0, p1=1.0, specials=("nan",),
+                  special_rate=rate)
+    x = _view(_gen(oracle, [s], 4 * n), 0, "f32", n)
+    k = int(np.isnan(x).sum())
+    if rate == 1.0:
+        assert k == n
+    else:
+        assert abs(k - rate * n) < 5 * math.sqrt(n * rate * (1 - rate)) + 1
+
+
+@pytest.mark.parametrize("dist", ["uniform", "normal"])
+def test_special_selection_is_independent_of_the_value(oracle, dist):
+    # the selection draws from its own purpose: the base values at selected
+    # positions follow the same law as all base values (two-sample KS)
+    from scipy import stats
+    n = 1 << 18
+    kw = dict(p0=-1.0, p1=1.0) if dist == "uniform" else dict(p0=0.0, p1=1.0)
+    base = W.GenSpec("f32", dist, n, seed=11, stream=4, ref_offset=0, **kw)
+    a = _view(_gen(oracle, [base], 4 * n), 0, "f32", n)
+    b = _view(_gen(oracle, [base.replace(specials=("nan",), special_rate=0.02)], 4 * n), 0, "f32", n)
+    sel = np.isnan(b)
+    assert abs(sel.sum() - 0.02 * n) < 5 * math.sqrt(n * 0.02 * 0.98)
+    assert stats.ks_2samp(a[sel], a[~sel]).pvalue > 1e-4
+    assert np.array_equal(a[~sel], b[~sel])
+
+
+def test_special_selection_word_layout(oracle):
+    # the documented selection: element g is special iff word g%4 of its
+    # SPECIAL_SEL block g/4 is below floor(rate 2^32)
+    n = 4096
+    rate = 0.05
+    s = W.GenSpec("f32", "uniform", n, seed=21, stream=6, ref_offset=0, p0=0.0, p1=1.0, specials=("nan",),
+                  special_rate=rate)
+    x = _view(_gen(oracle, [s], 4 * n), 0, "f32", n)
+    thr = math.floor(rate * 2 ** 32)
+    want = np.zeros(n, bool)
+    for b in range(n // 4):
+        w = oracle.draw(21, 6, "special_sel", b)
+        for j in range(4):
+            want[4 * b + j] = w[j] < thr
+    assert np.array_equal(np.isnan(x), want)
+
+
 def test_special_selection_does_not_move_base_values(oracle):
     # each purpose draws from its own stream: changing the rate keeps the
     # non-special elements bit-identical
