@@ -235,9 +235,9 @@ def reference_arm(args, rank, world):
     value = nbytes * args.steps / tot / 1e9
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": workload_dtype(args.workload),
             "data": "synthetic (seeded counter-based specs)",
-            "config": {"workload": wl.name, "sample": sample},
+            "config": {"workload": full_workload(args.workload).name, "sample": sample},
             "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -248,6 +248,12 @@ def reference_arm(args, rank, world):
 # ---------------------------------------------------------------------------
 def full_workload(name):
     return W.FULL_SIZE[name]()
+
+
+def workload_dtype(name):
+    """The element type the workload's arithmetic runs on."""
+    return {"ladder": "f32", "fp32_pair": "f32", "segmented": "mixed f32/f16/bf16/i32", "dotlike_bf16": "bf16",
+            "perm_i64": "int64"}[name]
 
 
 def ours_arm(args, rank, world):
@@ -420,8 +426,7 @@ def ours_arm(args, rank, world):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "f32" if args.workload in ("ladder", "fp32_pair") else
-                 {"segmented": "mixed f32/f16/bf16/i32", "dotlike_bf16": "bf16", "perm_i64": "int64"}[args.workload],
+        "dtype": workload_dtype(args.workload),
         "data": "synthetic (seeded counter-based specs)",
         "config": {"workload": wl.name, "synth_bytes_per_step": synth_b, "verified_bytes_per_step": verify_b,
                    "stages_run": stages_run,
