@@ -472,12 +472,32 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
   const size_t tb = pair_table_bytes(n_pairs);
   if (!ws_ok(d_ws, ws_bytes, tb + compare_partial_bytes(pairs, n_pairs))) return SV_EWORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  // many small segments go to one warp-per-segment launch (group key kSmallKey),
+  // the rest to one launch per dtype
+  constexpr uint32_t kSmallKey = 8;
+  int n_small = 0;
+  for (int i = 0; i < n_pairs; ++i) n_small += cmp_vectors(pairs[i]) <= kSmallVectors;
+  const bool split = n_small >= kSmallMinPairs;
   std::vector<int> order;
   std::vector<Group> groups;
-  group_by(n_pairs, [&](int i) { return pairs[i].dtype; }, order, groups);
+  group_by(n_pairs, [&](int i) {
+    return split && cmp_vectors(pairs[i]) <= kSmallVectors ? kSmallKey : pairs[i].dtype;
+  }, order, groups);
   HostTable<DevPair> tab(n_pairs, tb != 0);
   uint64_t slot_base = 0;
   for (Group& g : groups) {
+    if (g.key == kSmallKey) {  // one slot each; the combine reads just slot0
+      for (int k = g.begin; k < g.end; ++k) {
+        DevPair& d = tab[k];
+        d.p = pairs[order[k]];
+        d.work_begin = 0;
+        d.chunk = ~0ull >> 1;
+        d.slot0 = slot_base++;
+        d.orig = (uint32_t)order[k];
+        d.pad = 0;
+      }
+      continue;
+    }
     for (int k = g.begin; k < g.end; ++k) {
       g.tiles += cmp_tiles(pairs[order[k]]);
       g.units += cmp_units(pairs[order[k]]);
@@ -506,8 +526,12 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
   const uint8_t* cand = static_cast<const uint8_t*>(d_cand);
   const uint8_t* ref = static_cast<const uint8_t*>(d_ref);
   for (const Group& g : groups) {
-    const cudaError_t e = launch_compare_group(g.key, tab.data() + g.begin, dev ? dev + g.begin : nullptr,
-                                               g.end - g.begin, g.units, g.sh, cand, ref, partials, nullptr, st);
+    const DevPair* h = tab.data() + g.begin;
+    const DevPair* d = dev ? dev + g.begin : nullptr;
+    const cudaError_t e = g.key == kSmallKey
+                              ? launch_compare_small(h, d, g.end - g.begin, cand, ref, partials, st)
+                              : launch_compare_group(g.key, h, d, g.end - g.begin, g.units, g.sh, cand, ref, partials,
+                                                     nullptr, st);
     if (e != cudaSuccess) return SV_ECUDA;
   }
   return status_of(launch_combine(tab.data(), dev, n_pairs, partials, d_results, nullptr, 0, st));

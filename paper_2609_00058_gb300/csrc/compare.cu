@@ -282,23 +282,25 @@ __device__ void do_tail(Acc& a, const Tol& t, const uint8_t* xb, const uint8_t* 
 
 __device__ __forceinline__ uint4 ldg_stream(const uint4* p) { return __ldcs(p); }
 
-// elements [i0, i1) of one segment: i0 is tile-aligned, i1 a tile boundary or n
-template <int DT>
+// elements [i0, i1) of one segment by a team of NT threads (the CTA, or one
+// warp), `tid` the thread's rank in it: i0 is vector-aligned, i1 a loop
+// boundary or n
+template <int DT, int NT = kThreads>
 __device__ void cmp_run(Acc& a, const vc_pair& pr, const uint8_t* cand, const uint8_t* ref, uint64_t i0,
-                        uint64_t i1) {
+                        uint64_t i1, int tid = threadIdx.x) {
   constexpr uint32_t sz = elem_bytes(DT), VE = 16 / sz;
-  constexpr int U = kCmpTileBytes / 16 / kThreads;  // vectors per thread per tile (4)
+  constexpr int U = kCmpTileBytes / 16 / kThreads;  // vectors per thread per loop iteration (4)
   const Tol t{__double2float_rn(pr.atol), __double2float_rn(pr.rtol), (pr.flags & SV_EQUAL_NAN) != 0};
   const uint8_t* xb = cand + pr.cand_offset;
   const uint8_t* yb = ref + pr.ref_offset;
   const uint4* xv = reinterpret_cast<const uint4*>(xb);
   const uint4* yv = reinterpret_cast<const uint4*>(yb);
   const uint64_t v0 = i0 / VE, vfull = i1 / VE;  // whole vectors in [i0, i1)
-  for (uint64_t base = v0; base < vfull; base += (uint64_t)U * kThreads) {
+  for (uint64_t base = v0; base < vfull; base += (uint64_t)U * NT) {
     uint4 x[U], y[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const uint64_t v = base + (uint64_t)u * kThreads + threadIdx.x;
+      const uint64_t v = base + (uint64_t)u * NT + tid;
       if (v < vfull) {
         x[u] = ldg_stream(xv + v);
         y[u] = ldg_stream(yv + v);
@@ -307,7 +309,7 @@ __device__ void cmp_run(Acc& a, const vc_pair& pr, const uint8_t* cand, const ui
 
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const uint64_t v = base + (uint64_t)u * kThreads + threadIdx.x;
+      const uint64_t v = base + (uint64_t)u * NT + tid;
       if (v < vfull) do_vector<DT>(a, t, x[u], y[u], v * VE);
     }
     if constexpr (is_float(DT)) {
@@ -322,14 +324,12 @@ __device__ void cmp_run(Acc& a, const vc_pair& pr, const uint8_t* cand, const ui
     }
   }
   const uint64_t tail0 = vfull * VE;
-  if (tail0 < i1 && threadIdx.x == 0) do_tail<DT>(a, t, xb, yb, tail0, i1);
+  if (tail0 < i1 && tid == 0) do_tail<DT>(a, t, xb, yb, tail0, i1);
 }
 
-// block-wide fold of the accumulators into one partial (fixed order)
+// warp-wide fold of the accumulators (fixed order); the result is in lane 0
 template <bool FLOAT>
-__device__ void flush(Acc& a, Partial* out) {
-  __shared__ Partial wp[kThreads / 32];
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+__device__ __forceinline__ Partial warp_fold(const Acc& a) {
   uint64_t mism = a.mism, nan_d = a.nan_d, inf_d = a.inf_d, nonfin = a.nonfin, first = a.first;
   double ssq = a.ssq;
   uint64_t maxabs = FLOAT ? (uint64_t)__float_as_uint(a.maxabs_f) : a.maxabs_u;
@@ -347,7 +347,16 @@ __device__ void flush(Acc& a, Partial* out) {
     maxabs = m2 > maxabs ? m2 : maxabs;  // non-negative fp32 bits order like the values
     maxrel = fmax(maxrel, __shfl_down_sync(0xFFFFFFFFu, maxrel, o));
   }
-  if (lane == 0) wp[w] = Partial{mism, nan_d, inf_d, nonfin, first, ssq, maxabs, maxrel};
+  return Partial{mism, nan_d, inf_d, nonfin, first, ssq, maxabs, maxrel};
+}
+
+// block-wide fold of the accumulators into one partial (fixed order)
+template <bool FLOAT>
+__device__ void flush(Acc& a, Partial* out) {
+  __shared__ Partial wp[kThreads / 32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const Partial f = warp_fold<FLOAT>(a);
+  if (lane == 0) wp[w] = f;
   __syncthreads();
   if (threadIdx.x == 0) {
     Partial r = wp[0];
@@ -397,6 +406,38 @@ __global__ void __launch_bounds__(kThreads, 3) cmp_kernel(const __grid_constant_
     const uint64_t vlo = umax(u0, v_base), vhi = umin(u1, we);
     if (vhi > vlo) cmp_run<DT>(a, pr, p.cand, p.ref, (vlo - v_base) * VE, umin((vhi - v_base) * VE, pr.n));
     flush<is_float(DT)>(a, p.partials + cur.slot0 + blockIdx.x);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// many small segments (at most kSmallVectors vectors each): one warp per
+// segment, any dtype, no block barriers; the warp writes the segment's only
+// partial at its slot0 (the combine reads that one slot: work_begin 0 and a
+// chunk beyond the segment's units)
+// ---------------------------------------------------------------------------
+template <int DT>
+__device__ __forceinline__ void warp_segment(const vc_pair& pr, const uint8_t* cand, const uint8_t* ref, Partial* out,
+                                             int lane) {
+  Acc a;
+  acc_reset(a);
+  cmp_run<DT, 32>(a, pr, cand, ref, 0, pr.n, lane);
+  const Partial f = warp_fold<is_float(DT)>(a);
+  if (lane == 0) *out = f;
+}
+
+__global__ void __launch_bounds__(kThreads) cmp_small_kernel(const __grid_constant__ CmpParams p) {
+  const int w = (int)(blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5)), lane = threadIdx.x & 31;
+  if (w >= p.n) return;
+  const DevPair* dp = pentry(p, w);
+  const vc_pair& pr = dp->p;
+  Partial* out = p.partials + dp->slot0;
+  switch (pr.dtype) {  // uniform over the warp
+    case SV_F32: warp_segment<SV_F32>(pr, p.cand, p.ref, out, lane); break;
+    case SV_F16: warp_segment<SV_F16>(pr, p.cand, p.ref, out, lane); break;
+    case SV_BF16: warp_segment<SV_BF16>(pr, p.cand, p.ref, out, lane); break;
+    case SV_I32: warp_segment<SV_I32>(pr, p.cand, p.ref, out, lane); break;
+    case SV_I64: warp_segment<SV_I64>(pr, p.cand, p.ref, out, lane); break;
+    default: warp_segment<SV_U32>(pr, p.cand, p.ref, out, lane); break;
   }
 }
 
@@ -547,6 +588,23 @@ cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevP
     case SV_I64: cmp_kernel<SV_I64><<<sh.grid, kThreads, 0, st>>>(cp); break;
     default: cmp_kernel<SV_U32><<<sh.grid, kThreads, 0, st>>>(cp); break;
   }
+  count_launch();
+  return cudaGetLastError();
+}
+
+cudaError_t launch_compare_small(const DevPair* host, const DevPair* dev, int n, const uint8_t* cand,
+                                 const uint8_t* ref, Partial* partials, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  CmpParams cp;
+  fill_pairs(cp, host, dev, n);
+  cp.total = 0;
+  cp.chunk = 0;
+  cp.cand = cand;
+  cp.ref = ref;
+  cp.partials = partials;
+  cp.flag = nullptr;
+  const unsigned blocks = (unsigned)((n + kThreads / 32 - 1) / (kThreads / 32));
+  cmp_small_kernel<<<blocks, kThreads, 0, st>>>(cp);
   count_launch();
   return cudaGetLastError();
 }

@@ -128,6 +128,11 @@ LaunchShape compare_shape(uint32_t dtype, uint64_t units, uint64_t tiles);
 cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevPair* dev, int n, uint64_t units,
                                  LaunchShape sh, const uint8_t* cand, const uint8_t* ref, Partial* partials,
                                  const int32_t* flag, cudaStream_t st);
+// many small segments of any dtypes, one warp each (at most kSmallVectors vectors per segment)
+constexpr uint64_t kSmallVectors = 1024;
+constexpr int kSmallMinPairs = 64;  // below this many, small segments stay in their dtype groups
+cudaError_t launch_compare_small(const DevPair* host, const DevPair* dev, int n, const uint8_t* cand,
+                                 const uint8_t* ref, Partial* partials, cudaStream_t st);
 cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const Partial* partials,
                            vc_result* results, int32_t* flag, int first_group, cudaStream_t st);
 

@@ -94,7 +94,7 @@ def _segments(n_pairs, seed):
     return pairs, cand, ref
 
 
-@pytest.mark.parametrize("n_pairs,seed", [(1, 1), (5, 2), (8, 3), (9, 4), (64, 5), (700, 6)])
+@pytest.mark.parametrize("n_pairs,seed", [(1, 1), (5, 2), (8, 3), (9, 4), (64, 5), (200, 7), (700, 6)])
 def test_many_segments_mixed_dtypes(dev, n_pairs, seed):
     pairs, cand, ref = _segments(n_pairs, seed)
     got, want = run_both(dev, pairs, cand, ref)
