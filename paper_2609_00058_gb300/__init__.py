@@ -192,21 +192,9 @@ def to_c_pair(p) -> vc_pair:
 
 
 def _host_array(ctype, items):
-    """A ctypes array of `items`; tables longer than the kernel-parameter
-    capacity are placed in pinned (page-locked) host memory when a GPU is
-    present, so the library's copy of them to the device stays asynchronous."""
+    """A ctypes array of `items` in ordinary host memory (the library reads it
+    during the call and stages its own device table from pinned buffers)."""
     n = max(len(items), 1)
-    if len(items) > INLINE_ENTRIES:
-        try:
-            import torch
-            if torch.cuda.is_available():
-                buf = torch.empty(n * C.sizeof(ctype), dtype=torch.uint8, pin_memory=True)
-                arr = (ctype * n).from_address(buf.data_ptr())
-                for i, it in enumerate(items):
-                    arr[i] = it
-                return arr, buf
-        except (ImportError, RuntimeError):
-            pass
     return (ctype * n)(*items), None
 
 
