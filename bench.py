@@ -345,14 +345,13 @@ def ours_arm(args, rank, world):
     host = torch.empty(wl.arena_bytes, dtype=torch.uint8, pin_memory=True)
     host_res = torch.empty(results.numel(), dtype=torch.uint8, pin_memory=True)
     host_ff = torch.empty(1, dtype=torch.int32, pin_memory=True)
-    out_ranges = [(s.ref_offset, s.n * W.DTYPE_BYTES[s.dtype]) for c in wl.gen_calls for s in c
-                  if s.ref_offset is not None] + \
-                 [(s.cand_offset, s.n * W.DTYPE_BYTES[s.dtype]) for c in wl.gen_calls for s in c
-                  if s.cand_offset is not None]
-    d2h = sum(n for _, n in out_ranges) + host_res.numel() + (4 if wl.progressive else 0)
+    # the whole arena (every output array and the few alignment gaps between
+    # them) goes back, in large pieces rather than one copy per array
+    out_ranges = [(0, wl.arena_bytes)]
+    d2h = wl.arena_bytes + host_res.numel() + (4 if wl.progressive else 0)
     h2d = sum(C.n * ctypes.sizeof(sv.syn_spec) for C in spec_tabs) + pair_tab.n * ctypes.sizeof(sv.vc_pair)
 
-    # the outputs go to pinned host memory in pieces of at most 64 MiB spread
+    # the arena goes to pinned host memory in pieces of at most 64 MiB spread
     # over four copy streams (several copy engines at once); the verify runs
     # beside them on the compute stream, as both only read the arena
     copy_streams = [torch.cuda.Stream(dev) for _ in range(4)]
