@@ -39,11 +39,12 @@ METRIC = "verified GB/s and synthesized GB/s on 1 GB300, as % of HBM peak"
 L2_BYTES = 129 * 1000 * 1000  # GB300 L2 (bytes, nominal 129 MB)
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # dram bytes per launch of the dominant kernel from one ncu capture, keyed by
-# a hash of the kernel sources they were taken on (None once the code moves on)
+# a hash of the generator's sources they were taken on (None once they change)
 NCU_TRAFFIC = {
-    # gen_kernel<f32, normal>: 99,840 B read + 1,315,961,856 B written (no fixup launch:
-    # the one exact-count edit is applied by the generating CTA)
-    ("ladder", "923b349414480369"): 1316061696,
+    # gen_kernel<f32, normal>, median of the 7 launches of one single-pass ncu launch
+    # list (profiles/launches_ladder.md): 113,408 B read + 1,313,042,432 B written; no
+    # fixup launch (the one exact-count edit is applied by the generating CTA)
+    ("ladder", "c0f97f807977535d"): 1313155840,
 }
 
 
@@ -107,11 +108,10 @@ def alu_floor_s(wl, peaks):
 
 
 def source_hash():
+    """Hash of the generator's kernel sources (the roofline's kernel)."""
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2609_00058_gb300", "csrc")
-    for f in sorted(os.listdir(d)):
-        if not f.endswith((".cu", ".cuh", ".h")):
-            continue
+    for f in ("generate.cu", "sv_device.cuh", "sv_kernels.h"):
         with open(os.path.join(d, f), "rb") as fh:
             h.update(f.encode() + fh.read())
     return h.hexdigest()[:16]
