@@ -77,9 +77,6 @@ __device__ __forceinline__ void store4(uint8_t* base, uint64_t i, const typename
   }
 }
 
-#ifndef SV_GEN_QPI
-#define SV_GEN_QPI 1  // quanta per thread per iteration (independent Philox chains)
-#endif
 #ifndef SV_GEN_MINB
 #define SV_GEN_MINB 2  // resident CTAs per SM the register budget must allow
 #endif
@@ -141,54 +138,58 @@ __device__ __noinline__ void fused_edits(const Ctx& c, const syn_spec& s, uint64
   else reinterpret_cast<T*>(cand)[g - s.elem_offset] = (T)bits;
 }
 
-// elements [i0, i1) of one spec, by 4-element quanta spread over the CTA.
-// `cold` is the spec's context in shared memory; the hot fields are copied to
-// registers.  Each thread carries QPI quanta at once so their Philox and
-// Box-Muller chains overlap; a quantum past the end recomputes the last one
-// and is not stored.
-template <int DT, int DIST, int QPI>
+// base values and special values of the quantum g .. g+3
+template <int DT, int DIST>
+__device__ __forceinline__ void gen_quantum(const Ctx& c, const Ctx& cold, uint64_t g, typename Store<DT>::T v[4]) {
+  if (one_block_dist<DT, DIST>() && c.sp_thr) {
+    // the quantum's VALUE and SPECIAL_SEL blocks as two interleaved chains
+    const uint64_t blk = g >> 2;
+    uint4 wv = make_uint4((uint32_t)blk, (uint32_t)(blk >> 32), c.stream, P_VALUE);
+    uint4 ws = make_uint4((uint32_t)blk, (uint32_t)(blk >> 32), c.stream, P_SPECIAL_SEL);
+    philox2_rk(wv, ws, c.rk);
+    base4_words<DT, DIST>(c, wv, v);
+    specials4_words<DT, DIST>(c, cold, g, ws, v);
+  } else {
+    base4<DT, DIST>(c, g, v);
+    if (c.sp_thr) specials4<DT, DIST>(c, cold, g, v);
+  }
+}
+
+// the clean output and, after the element-wise perturbation, the twin
+template <int DT>
+__device__ __forceinline__ void store_quantum(const Ctx& c, const Ctx& cold, uint8_t* ref, uint8_t* cand, uint64_t g,
+                                              uint64_t i, typename Store<DT>::T v[4], uint32_t valid) {
+  if (ref) store4<DT>(ref, i, v, valid);
+  if (cand) {
+    if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, cold, g, v);
+    store4<DT>(cand, i, v, valid);
+  }
+}
+
+// elements [i0, i1) of one spec, by 4-element quanta spread over the CTA:
+// the full quanta in a loop with no per-quantum bounds, then at most one
+// ragged last quantum.  `cold` is the spec's context in shared memory; the
+// hot fields are copied to registers.
+template <int DT, int DIST>
 __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_t i1, uint8_t* arena) {
   using T = typename Store<DT>::T;
   const Ctx c = cold;
   uint8_t* ref = s.ref_offset == SV_NO_OUTPUT ? nullptr : arena + s.ref_offset;
   uint8_t* cand = s.cand_offset == SV_NO_OUTPUT ? nullptr : arena + s.cand_offset;
   const uint64_t eo = s.elem_offset, n = s.n;
-  const uint64_t q0 = i0 >> 2, q1 = (i1 + 3) >> 2;
-  for (uint64_t q = q0 + threadIdx.x; q < q1; q += (uint64_t)QPI * kThreads) {
-    T v[QPI][4];
-    uint64_t qu[QPI];
-#pragma unroll
-    for (int u = 0; u < QPI; ++u) qu[u] = umin(q + (uint64_t)u * kThreads, q1 - 1);
-    if (one_block_dist<DT, DIST>() && c.sp_thr) {
-      // the quantum's VALUE and SPECIAL_SEL blocks as two interleaved chains
-#pragma unroll
-      for (int u = 0; u < QPI; ++u) {
-        const uint64_t g = eo + (qu[u] << 2), blk = g >> 2;
-        uint4 wv = make_uint4((uint32_t)blk, (uint32_t)(blk >> 32), c.stream, P_VALUE);
-        uint4 ws = make_uint4((uint32_t)blk, (uint32_t)(blk >> 32), c.stream, P_SPECIAL_SEL);
-        philox2_rk(wv, ws, c.rk);
-        base4_words<DT, DIST>(c, wv, v[u]);
-        specials4_words<DT, DIST>(c, cold, g, ws, v[u]);
-      }
-    } else {
-#pragma unroll
-      for (int u = 0; u < QPI; ++u) base4<DT, DIST>(c, eo + (qu[u] << 2), v[u]);
-      if (c.sp_thr) {
-#pragma unroll
-        for (int u = 0; u < QPI; ++u) specials4<DT, DIST>(c, cold, eo + (qu[u] << 2), v[u]);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < QPI; ++u) {
-      if (q + (uint64_t)u * kThreads >= q1) break;
-      const uint64_t i = qu[u] << 2;
-      const uint32_t valid = (uint32_t)umin(4, n - i);
-      if (ref) store4<DT>(ref, i, v[u], valid);
-      if (cand) {
-        if (c.pe_kind != SV_PERT_NONE) pelem4<DT>(c, cold, eo + i, v[u]);
-        store4<DT>(cand, i, v[u], valid);
-      }
-    }
+  const uint64_t q0 = i0 >> 2, q1 = (i1 + 3) >> 2, qfull = umin(q1, n >> 2);
+  uint64_t q = q0 + threadIdx.x;
+  for (; q < qfull; q += kThreads) {
+    T v[4];
+    const uint64_t i = q << 2;
+    gen_quantum<DT, DIST>(c, cold, eo + i, v);
+    store_quantum<DT>(c, cold, ref, cand, eo + i, i, v, 4);
+  }
+  if (q < q1) {  // the last quantum of the spec, with n % 4 elements
+    T v[4];
+    const uint64_t i = q << 2;
+    gen_quantum<DT, DIST>(c, cold, eo + i, v);
+    store_quantum<DT>(c, cold, ref, cand, eo + i, i, v, (uint32_t)(n - i));
   }
 }
 
@@ -217,7 +218,7 @@ __global__ void __launch_bounds__(kThreads, SV_GEN_MINB) gen_kernel(const __grid
     if (threadIdx.x == 0) ctx = make_ctx(cur.s, p.arena);
     __syncthreads();
     const uint64_t i0 = (lo - q_base) * 4, i1 = umin((hi - q_base) * 4, cur.s.n);
-    gen_run<DT, DIST, SV_GEN_QPI>(ctx, cur.s, i0, i1, p.arena);
+    gen_run<DT, DIST>(ctx, cur.s, i0, i1, p.arena);
     if (cur.fused) {  // uniform: the spec's exact-count edits inside this CTA's range
       __syncthreads();
       fused_edits<DT, DIST>(ctx, cur.s, cur.s.elem_offset + i0, cur.s.elem_offset + i1, p.arena);
@@ -524,7 +525,7 @@ static void fill_params(GenParams& gp, const DevSpec* host, const DevSpec* dev, 
 
 LaunchShape generate_shape(uint32_t dtype, uint32_t dist, uint64_t units, uint64_t tiles) {
   const void* k = gen_kernel_for(dtype, dist);
-  return shape_for(units, tiles, k ? grid_cap_for(k) : 1, (uint64_t)SV_GEN_QPI * kThreads);
+  return shape_for(units, tiles, k ? grid_cap_for(k) : 1, (uint64_t)kThreads);
 }
 
 cudaError_t launch_generate_group(uint32_t dtype, uint32_t dist, const DevSpec* host, const DevSpec* dev, int n,
