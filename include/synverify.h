@@ -71,10 +71,16 @@ enum { SV_F32 = 0, SV_F16 = 1, SV_BF16 = 2, SV_I32 = 3, SV_I64 = 4, SV_U32 = 5 }
  *                  (written by an earlier call).  cols % 4 == 0.
  *   SV_RAW_BITS    the words themselves (16-bit types: the word's top half).
  *   SV_CONSTANT    p0 (float types) or i0 (integer types) everywhere.
+ *   SV_FROM_ARENA  any type: element g of the existing array of logical_n
+ *                  elements of the same type at a_offset of the same arena
+ *                  (written earlier; 16-byte aligned; must not overlap this
+ *                  spec's outputs).  Special values and perturbations apply
+ *                  as to drawn values, so an existing output (a trusted
+ *                  reference's, say) gets perturbed twins.
  */
 enum {
   SV_UNIFORM = 0, SV_NORMAL = 1, SV_INT_RANGE = 2, SV_PERMUTATION = 3,
-  SV_DOTLIKE = 4, SV_RAW_BITS = 5, SV_CONSTANT = 6
+  SV_DOTLIKE = 4, SV_RAW_BITS = 5, SV_CONSTANT = 6, SV_FROM_ARENA = 7
 };
 
 /* ---- special values (syn_spec.special_mask, OR of these) ----
@@ -143,7 +149,7 @@ typedef struct sv_perturb {
  * generating an array in chunks gives the same bytes as generating it whole. */
 typedef struct syn_spec {
   uint32_t dtype;        /* SV_F32 ... SV_U32 */
-  uint32_t dist;         /* SV_UNIFORM ... SV_CONSTANT */
+  uint32_t dist;         /* SV_UNIFORM ... SV_FROM_ARENA */
   uint64_t n;            /* elements written per output */
   uint64_t seed;         /* Philox key */
   uint32_t stream;       /* Philox counter word 2 of base and special draws */
@@ -156,7 +162,7 @@ typedef struct syn_spec {
   double p0, p1;         /* float parameters (see SV_UNIFORM ...) */
   int64_t i0, i1;        /* integer parameters */
   uint64_t rows, cols, dot_k;  /* SV_DOTLIKE shape */
-  uint64_t a_offset, b_offset; /* SV_DOTLIKE factors, multiples of 16 */
+  uint64_t a_offset, b_offset; /* SV_DOTLIKE factors / SV_FROM_ARENA source (a_offset), multiples of 16 */
   sv_perturb pelem;      /* NONE, RATE_ADD_PM or REL_NOISE */
   sv_perturb pcount;     /* NONE, COUNT_SET, COUNT_ADD or SWAP_PAIRS */
 } syn_spec;

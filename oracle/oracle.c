@@ -349,6 +349,12 @@ static uint64_t base_value(const or_spec* s, const uint8_t* arena, uint64_t g) {
       if (elem_bytes(dt) == 2) return w[g & 3] >> 16;
       return w[g & 3];
     }
+    case OR_FROM_ARENA: {
+      /* element g of the existing array at a_offset (same element type) */
+      uint64_t bits = 0;
+      memcpy(&bits, arena + s->a_offset + g * elem_bytes(dt), elem_bytes(dt)); /* little-endian */
+      return bits;
+    }
     case OR_CONSTANT:
     default:
       if (is_float_dtype(dt)) return store_f32(dt, (float)s->p0);
@@ -496,7 +502,7 @@ int or_check_spec(const or_spec* s, uint64_t arena_bytes) {
   switch (s->dist) {
     case OR_UNIFORM: case OR_NORMAL: case OR_DOTLIKE: if (!fl) return -1; break;
     case OR_INT_RANGE: case OR_PERMUTATION: if (!is_int_dtype(dt)) return -1; break;
-    case OR_RAW_BITS: case OR_CONSTANT: break;
+    case OR_RAW_BITS: case OR_CONSTANT: case OR_FROM_ARENA: break;
     default: return -1;
   }
   if (s->ref_offset == OR_ABSENT && s->cand_offset == OR_ABSENT) return -1;
@@ -514,6 +520,16 @@ int or_check_spec(const or_spec* s, uint64_t arena_bytes) {
     if (s->cols == 0 || s->rows * s->cols != N || s->dot_k == 0) return -1;
     if (s->a_offset + 4 * s->rows * s->dot_k > arena_bytes) return -1;
     if (s->b_offset + 4 * s->dot_k * s->cols > arena_bytes) return -1;
+  }
+  if (s->dist == OR_FROM_ARENA) {
+    /* the source is the whole logical array; it must lie in the arena, away from the outputs */
+    uint64_t src = N * elem_bytes(dt);
+    if (s->a_offset % 16 || s->a_offset > arena_bytes || src > arena_bytes - s->a_offset) return -1;
+    if (s->ref_offset != OR_ABSENT && bytes && s->ref_offset < s->a_offset + src && s->a_offset < s->ref_offset + bytes)
+      return -1;
+    if (s->cand_offset != OR_ABSENT && bytes && s->cand_offset < s->a_offset + src &&
+        s->a_offset < s->cand_offset + bytes)
+      return -1;
   }
   uint32_t fmask = OR_SP_NAN | OR_SP_PINF | OR_SP_NINF | OR_SP_DENORM | OR_SP_ZERO | OR_SP_DUP;
   uint32_t imask = OR_SP_ZERO | OR_SP_IMIN | OR_SP_IMAX | OR_SP_DUP;

@@ -37,7 +37,7 @@ enum { OR_F32 = 0, OR_F16 = 1, OR_BF16 = 2, OR_I32 = 3, OR_I64 = 4, OR_U32 = 5 }
 /* base value distributions */
 enum {
   OR_UNIFORM = 0, OR_NORMAL = 1, OR_INT_RANGE = 2, OR_PERMUTATION = 3,
-  OR_DOTLIKE = 4, OR_RAW_BITS = 5, OR_CONSTANT = 6
+  OR_DOTLIKE = 4, OR_RAW_BITS = 5, OR_CONSTANT = 6, OR_FROM_ARENA = 7
 };
 /* special-value kinds (bit positions of the mask, drawn in ascending order) */
 enum {

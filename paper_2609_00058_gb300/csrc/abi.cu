@@ -88,7 +88,7 @@ static int check_range(uint64_t off, uint64_t bytes, uint64_t buf) {
 static bool valid_rate(double r) { return r >= 0.0 && r <= 1.0; }  // false for NaN
 
 static int check_spec(const syn_spec& s, uint64_t arena) {
-  if (s.dtype > SV_U32 || s.dist > SV_CONSTANT) return SV_EINVAL;
+  if (s.dtype > SV_U32 || s.dist > SV_FROM_ARENA) return SV_EINVAL;
   const bool fl = is_float((int)s.dtype);
   switch (s.dist) {
     case SV_UNIFORM: case SV_NORMAL: case SV_DOTLIKE: if (!fl) return SV_EINVAL; break;
@@ -127,7 +127,14 @@ static int check_spec(const syn_spec& s, uint64_t arena) {
     if (s.rows > (1ull << 40) / s.dot_k || s.cols > (1ull << 40) / s.dot_k) return SV_ERANGE;
     if ((rc = check_range(s.a_offset, 4 * s.rows * s.dot_k, arena))) return rc;
     if ((rc = check_range(s.b_offset, 4 * s.dot_k * s.cols, arena))) return rc;
-    if ((s.rows + 63) / 64 > 65535) return SV_ERANGE;  // grid.y of the tiled kernel
+  }
+  if (s.dist == SV_FROM_ARENA) {  // the source: the whole logical array, apart from the outputs
+    const uint64_t src = N * elem_bytes((int)s.dtype);
+    if ((rc = check_range(s.a_offset, src, arena))) return rc;
+    auto overlaps = [&](uint64_t off) {
+      return off != SV_NO_OUTPUT && bytes && src && off < s.a_offset + src && s.a_offset < off + bytes;
+    };
+    if (overlaps(s.ref_offset) || overlaps(s.cand_offset)) return SV_EINVAL;
   }
   const sv_perturb& pe = s.pelem;
   if (pe.kind != SV_PERT_NONE && pe.kind != SV_PERT_RATE_ADD_PM && pe.kind != SV_PERT_REL_NOISE) return SV_EINVAL;

@@ -233,7 +233,9 @@ __global__ void __launch_bounds__(kThreads, SV_GEN_MINB) gen_kernel(const __grid
   X(SV_BF16, SV_UNIFORM) X(SV_BF16, SV_NORMAL) X(SV_BF16, SV_RAW_BITS) X(SV_BF16, SV_CONSTANT)     \
   X(SV_I32, SV_INT_RANGE) X(SV_I32, SV_PERMUTATION) X(SV_I32, SV_RAW_BITS) X(SV_I32, SV_CONSTANT)  \
   X(SV_U32, SV_INT_RANGE) X(SV_U32, SV_PERMUTATION) X(SV_U32, SV_RAW_BITS) X(SV_U32, SV_CONSTANT)  \
-  X(SV_I64, SV_INT_RANGE) X(SV_I64, SV_PERMUTATION) X(SV_I64, SV_RAW_BITS) X(SV_I64, SV_CONSTANT)
+  X(SV_I64, SV_INT_RANGE) X(SV_I64, SV_PERMUTATION) X(SV_I64, SV_RAW_BITS) X(SV_I64, SV_CONSTANT)             \
+  X(SV_F32, SV_FROM_ARENA) X(SV_F16, SV_FROM_ARENA) X(SV_BF16, SV_FROM_ARENA) X(SV_I32, SV_FROM_ARENA)         \
+  X(SV_U32, SV_FROM_ARENA) X(SV_I64, SV_FROM_ARENA)
 
 static const void* gen_kernel_for(uint32_t dtype, uint32_t dist) {
   switch (SV_COMBO(dtype, dist)) {
@@ -293,6 +295,8 @@ __device__ void fix_dispatch(const Ctx& c, const syn_spec& s, uint64_t u, uint8_
     SV_CASE(SV_U32, SV_CONSTANT)
     SV_CASE(SV_I64, SV_INT_RANGE) SV_CASE(SV_I64, SV_PERMUTATION) SV_CASE(SV_I64, SV_RAW_BITS)
     SV_CASE(SV_I64, SV_CONSTANT)
+    SV_CASE(SV_F32, SV_FROM_ARENA) SV_CASE(SV_F16, SV_FROM_ARENA) SV_CASE(SV_BF16, SV_FROM_ARENA)
+    SV_CASE(SV_I32, SV_FROM_ARENA) SV_CASE(SV_U32, SV_FROM_ARENA) SV_CASE(SV_I64, SV_FROM_ARENA)
 #undef SV_CASE
     default: break;
   }

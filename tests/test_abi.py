@@ -93,6 +93,10 @@ BAD_SPECS = [
     (dict(dtype="bf16", dist="dotlike", rows=4, cols=8, dot_k=8, n=24), -1),   # rows*cols != n
     (dict(dtype="bf16", dist="dotlike", rows=4, cols=8, dot_k=8, n=32, a_offset=8), -2),
     (dict(dtype="bf16", dist="dotlike", rows=4, cols=8, dot_k=8, n=32, b_offset=16256), -3),
+    (dict(dtype="i32", dist="from_arena", n=256, a_offset=8192 + 8), -2),       # misaligned source
+    (dict(dtype="i32", dist="from_arena", n=256, a_offset=16384 - 512), -3),    # source past the arena
+    (dict(dtype="i32", dist="from_arena", n=256, a_offset=512), -1),            # source overlaps the output
+    (dict(dtype="i32", dist="from_arena", n=256, a_offset=8192, logical_n=4096), -3),  # source of N elements
 ]
 
 
@@ -109,7 +113,9 @@ def test_valid_specs_accepted(lib):
     ok = [_spec(), _spec(dtype="bf16", dist="normal", p0=5.0, p1=10.0, specials=("nan", "dup"), special_rate=0.1),
           _spec(dtype="i64", dist="permutation", n=512, specials=("imin", "imax"), special_rate=0.01,
                 pcount=W.Perturb("swap_pairs", count=17)),
-          _spec(dtype="bf16", dist="dotlike", rows=4, cols=8, dot_k=8, n=32, a_offset=256, b_offset=512)]
+          _spec(dtype="bf16", dist="dotlike", rows=4, cols=8, dot_k=8, n=32, a_offset=256, b_offset=512),
+          _spec(dtype="i64", dist="from_arena", n=256, a_offset=8192, specials=("dup",), special_rate=0.1,
+                pcount=W.Perturb("count_add", count=3, ivalue=1))]
     for s in ok:
         assert sv.check_specs([s], 4096 * 4) == 0
 

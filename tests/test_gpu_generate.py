@@ -318,3 +318,44 @@ def test_zero_length_and_single_element(dev):
              W.GenSpec("bf16", "normal", 1, ref_offset=768, p0=0, p1=1, specials=("nan",), special_rate=1.0)]
     g, h = gen_both(dev, [specs], 1024)
     assert np.array_equal(g, h)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f16", "bf16", "i32", "u32", "i64"])
+def test_from_arena_matches_oracle(dev, dtype):
+    # base values read from an existing array of N = 3 * 8192 + 13 elements
+    # (its last quantum is ragged: the kernel must not read past it), with
+    # specials, an element-wise and an exact-count perturbation; then a chunk
+    # that ends at the array's end
+    import torch
+    n = 3 * 8192 + 13
+    sz = W.DTYPE_BYTES[dtype]
+    ar = W.Arena()
+    src_off, ref_off, cand_off = ar.take(n * sz), ar.take(n * sz), ar.take(n * sz)
+    h = np.zeros(ar.size, np.uint8)
+    rng = np.random.default_rng(17)
+    if dtype in W.FLOAT_DTYPES:
+        f = rng.normal(0.0, 3.0, n).astype(np.float32)
+        bits = f.view(np.uint32) if dtype == "f32" else (
+            oracle.f32_to_bf16(f) if dtype == "bf16" else oracle.f32_to_f16(f))
+        specials, pelem = ("nan", "pinf", "denorm", "dup"), W.Perturb("rel_noise", stream=3, value=2.0 ** -9)
+        pcount = W.Perturb("count_add", stream=4, count=5, value=0.5)
+    else:
+        bits = rng.integers(0, 1 << 63, n, dtype=np.uint64).astype({4: np.uint32, 8: np.uint64}[sz])
+        specials, pelem = ("zero", "imin", "dup"), W.Perturb("rate_add_pm", stream=3, rate=0.01, ivalue=7)
+        pcount = W.Perturb("swap_pairs", stream=4, count=5)
+    h[src_off: src_off + n * sz] = np.ascontiguousarray(bits).view(np.uint8)
+    spec = W.GenSpec(dtype, "from_arena", n, seed=31, stream=2, ref_offset=ref_off, cand_offset=cand_off,
+                     a_offset=src_off, specials=specials, special_rate=0.01, pelem=pelem, pcount=pcount)
+    for specs in ([spec], [spec.replace(n=n - 8192, elem_offset=8192, logical_n=n, ref_offset=ref_off + 8192 * sz,
+                                        cand_offset=cand_off + 8192 * sz)]):
+        want = h.copy()
+        oracle.generate(specs, want)
+        a = torch.from_numpy(h.copy()).to(dev)
+        sv.generate(specs, a)
+        got = a.cpu().numpy()
+        s0 = specs[0]
+        if dtype in W.FLOAT_DTYPES:  # the noise runs Box-Muller: compare as the other parity tests do
+            check_spec_outputs(got, want, s0)
+            assert np.array_equal(got[:ref_off], want[:ref_off])  # the source is untouched
+        else:
+            assert np.array_equal(got, want), dtype

@@ -336,3 +336,45 @@ def test_workload_perm_small(oracle):
     _, res, _ = oracle.run_workload(wl)
     r = res[0]
     assert 0 < r["mismatches"] <= 34 and r["mismatches"] % 2 == 0
+
+
+@pytest.mark.parametrize("dtype", ["i32", "i64", "f32", "bf16"])
+def test_from_arena_copies_the_source_and_applies_specials(oracle, dtype):
+    # base values read from an existing array; specials (zero, duplicates of
+    # the source) and an exact-count edit on top; a chunked run matches
+    n = 5001
+    sz = W.DTYPE_BYTES[dtype]
+    rng = np.random.default_rng(3)
+    src_off, ref_off, cand_off = 0, 32768 * sz // 4 * 4, 65536 * sz // 4 * 4
+    size = cand_off + n * sz + 256
+    arena = np.zeros(size, np.uint8)
+    src = rng.integers(1, 1 << (8 * min(sz, 4)), n, dtype=np.uint64).astype({2: np.uint16, 4: np.uint32,
+                                                                            8: np.uint64}[sz])
+    if dtype in ("f32", "bf16"):  # finite, nonzero floats
+        f = rng.uniform(1.0, 2.0, n).astype(np.float32)
+        src = f.view(np.uint32) if dtype == "f32" else (f.view(np.uint32) >> 16).astype(np.uint16)
+    arena[src_off: src_off + n * sz] = src.view(np.uint8)
+    pc = W.Perturb("count_add", stream=2, count=3, value=1.0, ivalue=5)
+    spec = W.GenSpec(dtype, "from_arena", n, seed=9, stream=1, ref_offset=ref_off, cand_offset=cand_off,
+                     a_offset=src_off, specials=("zero", "dup"), special_rate=0.05, pcount=pc)
+    assert oracle.check_spec(spec, size) == 0
+    whole = arena.copy()
+    oracle.generate([spec], whole)
+    ut = {2: np.uint16, 4: np.uint32, 8: np.uint64}[sz]  # compare bit patterns
+    src = src.view(ut)
+    ref = _view(whole, ref_off, dtype, n).view(ut)
+    cand = _view(whole, cand_off, dtype, n).view(ut)
+    keep = ref == src
+    special = ~keep
+    assert 0.03 * n < special.sum() < 0.07 * n
+    srcset = set(src.tolist())
+    assert all(v == 0 or v in srcset for v in ref[special].tolist())  # zero or a duplicate
+    assert 1 <= np.count_nonzero(cand != ref) <= 3
+    assert np.array_equal(_view(whole, src_off, dtype, n).view(ut), src)  # the source is untouched
+    # chunks of the same logical array give the same bytes
+    chunked = arena.copy()
+    cuts = [0, 1000, 2048, n]
+    parts = [spec.replace(n=c1 - c0, elem_offset=c0, logical_n=n, ref_offset=ref_off + c0 * sz,
+                          cand_offset=cand_off + c0 * sz) for c0, c1 in zip(cuts[:-1], cuts[1:])]
+    oracle.generate(parts, chunked)
+    assert np.array_equal(chunked, whole)

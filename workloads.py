@@ -8,7 +8,7 @@ descriptions while sharing no code with each other.
 
 Names are strings; each side maps them onto its own enumerations:
   dtypes        f32 f16 bf16 i32 i64 u32
-  dists         uniform normal int_range permutation dotlike raw_bits constant
+  dists         uniform normal int_range permutation dotlike raw_bits constant from_arena
   special kinds nan pinf ninf denorm zero imin imax dup
   perturbations none rate_add_pm rel_noise count_set count_add swap_pairs
 
