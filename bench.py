@@ -341,6 +341,28 @@ def ours_arm(args, rank, world):
     total_ms = sum(step_each) if flush is not None else start.elapsed_time(end)
     total_ms = max_over_ranks(total_ms, world)
 
+    # the dot-like workload's candidate pass alone: the noisy twin of the
+    # existing reference array (SV_FROM_ARENA + relative noise), the part of
+    # its synthesis that is not the dot product
+    cand_pass = None
+    if args.workload == "dotlike_bf16":
+        d = wl.gen_calls[1][0]
+        cp = sv.SpecTable([W.GenSpec(d.dtype, "from_arena", d.n, seed=d.seed, stream=d.stream, ref_offset=None,
+                                     cand_offset=d.cand_offset, a_offset=d.ref_offset, pelem=d.pelem)])
+        for _ in range(3):
+            sv.generate(cp, arena, workspace=ws)
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        c0.record(stream)
+        for _ in range(args.steps):
+            sv.generate(cp, arena, workspace=ws)
+        c1.record(stream)
+        torch.cuda.synchronize()
+        cp_ms = c0.elapsed_time(c1) / args.steps
+        cp_bytes = 2 * d.n * W.DTYPE_BYTES[d.dtype]  # reference read + candidate written
+        cand_pass = {"what": "candidate pass alone: reference read, noisy twin written", "ms": cp_ms,
+                     "bytes": cp_bytes, "gbs": cp_bytes / (cp_ms * 1e-3) / 1e9}
+
     # end to end: synthesized data delivered to pinned host buffers, verdicts read back
     host = torch.empty(wl.arena_bytes, dtype=torch.uint8, pin_memory=True)
     host_res = torch.empty(results.numel(), dtype=torch.uint8, pin_memory=True)
@@ -442,6 +464,7 @@ def ours_arm(args, rank, world):
         "step_ms_median": statistics.median(step_each),
         "step_ms_best": min(step_each),
         "roofline": roofline,
+        **({"candidate_pass": dict(cand_pass, frac_of_hbm=cand_pass["gbs"] / hbm)} if cand_pass else {}),
         "e2e": {"value": job_throughput(step_bytes, e2e_steps, world, e2e_s), "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps},
         "clocks": clocks,

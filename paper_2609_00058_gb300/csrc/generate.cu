@@ -179,15 +179,47 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
   const uint64_t eo = s.elem_offset, n = s.n;
   const uint64_t q0 = i0 >> 2, q1 = (i1 + 3) >> 2, qfull = umin(q1, n >> 2);
   uint64_t q = q0 + threadIdx.x;
-  for (; q < qfull; q += kThreads) {
-    T v[4];
-    const uint64_t i = q << 2;
-    gen_quantum<DT, DIST>(c, cold, eo + i, v);
-    store_quantum<DT>(c, cold, ref, cand, eo + i, i, v, 4);
+  if constexpr (DIST == SV_FROM_ARENA) {
+    // values read from memory, two quanta per iteration: their relative noise
+    // (the usual perturbation of such twins) runs as two interleaved chains
+    for (; q < qfull; q += 2ull * kThreads) {
+      const uint64_t q2 = q + kThreads, ia = q << 2, ib = q2 << 2;
+      const bool two = q2 < qfull;
+      T va[4], vb[4];
+      base4<DT, DIST>(c, eo + ia, va);
+      if (two) base4<DT, DIST>(c, eo + ib, vb);
+      if (c.sp_thr) {
+        specials4<DT, DIST>(c, cold, eo + ia, va);
+        if (two) specials4<DT, DIST>(c, cold, eo + ib, vb);
+      }
+      if constexpr (is_float(DT)) {
+        if (two && cand && c.pe_kind == SV_PERT_REL_NOISE) {
+          if (ref) {
+            store4<DT>(ref, ia, va, 4);
+            store4<DT>(ref, ib, vb, 4);
+          }
+          rel_noise4x2<DT>(c, eo + ia, va, eo + ib, vb);
+          store4<DT>(cand, ia, va, 4);
+          store4<DT>(cand, ib, vb, 4);
+          continue;
+        }
+      }
+      store_quantum<DT>(c, cold, ref, cand, eo + ia, ia, va, 4);
+      if (two) store_quantum<DT>(c, cold, ref, cand, eo + ib, ib, vb, 4);
+    }
+  } else {
+    for (; q < qfull; q += kThreads) {
+      T v[4];
+      const uint64_t i = q << 2;
+      gen_quantum<DT, DIST>(c, cold, eo + i, v);
+      store_quantum<DT>(c, cold, ref, cand, eo + i, i, v, 4);
+    }
   }
-  if (q < q1) {  // the last quantum of the spec, with n % 4 elements
+  // the spec's last quantum, with n % 4 elements, goes to the thread whose
+  // stride it falls on (q1 - 1 = n / 4 when it exists)
+  if (q1 > qfull && (q1 - 1 - q0) % kThreads == threadIdx.x) {
     T v[4];
-    const uint64_t i = q << 2;
+    const uint64_t i = (q1 - 1) << 2;
     gen_quantum<DT, DIST>(c, cold, eo + i, v);
     store_quantum<DT>(c, cold, ref, cand, eo + i, i, v, (uint32_t)(n - i));
   }

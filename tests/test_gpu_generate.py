@@ -359,3 +359,23 @@ def test_from_arena_matches_oracle(dev, dtype):
             assert np.array_equal(got[:ref_off], want[:ref_off])  # the source is untouched
         else:
             assert np.array_equal(got, want), dtype
+
+
+def test_candidate_pass_from_the_reference_equals_the_fused_twin(dev):
+    # the dot-like kernel writes the reference and its noisy twin together; the
+    # same twin made afterwards from the reference array (SV_FROM_ARENA with
+    # the same noise) is bit-identical
+    import torch
+    rows, cols, k = 200, 520, 64
+    wl = W.dotlike_bf16_pair(rows=rows, cols=cols, k=k)
+    n = rows * cols
+    extra = (2 * n + 255) // 256 * 256
+    a = torch.zeros(wl.arena_bytes + extra, dtype=torch.uint8, device=dev)
+    for call in wl.gen_calls:
+        sv.generate(call, a)
+    d = wl.gen_calls[1][0]
+    twin = W.GenSpec("bf16", "from_arena", n, seed=d.seed, stream=d.stream, ref_offset=None,
+                     cand_offset=wl.arena_bytes, a_offset=d.ref_offset, pelem=d.pelem)
+    sv.generate([twin], a)
+    h = a.cpu().numpy()
+    assert np.array_equal(h[d.cand_offset: d.cand_offset + 2 * n], h[wl.arena_bytes: wl.arena_bytes + 2 * n])
