@@ -294,6 +294,14 @@ int sv_abi_version(void);
  * work's launches.  Thread-safe; never fails. */
 uint64_t sv_kernel_launches(void);
 
+/* Test hook (no counterpart in the paper): the next n kernel launches of this
+ * library, on any device or stream, use an invalid launch configuration, so
+ * they fail at launch without running (no device fault; the context stays
+ * usable) and the calls that made them return SV_ECUDA.  Lets a caller's
+ * error handling be tested without a GPU fault.  n = 0 cancels; n < 0:
+ * SV_EINVAL.  Process-wide. */
+int sv_debug_fail_launches(int n);
+
 #ifdef __cplusplus
 }
 #endif

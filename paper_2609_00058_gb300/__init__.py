@@ -136,6 +136,7 @@ EXPORTS = [
     ("sv_abi_version", C.c_int, []),
     ("sv_kernel_launches", C.c_uint64, []),
     ("syn_box_muller", C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
+    ("sv_debug_fail_launches", C.c_int, [C.c_int]),
 ]
 
 _lib = None

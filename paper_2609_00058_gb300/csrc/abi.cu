@@ -46,6 +46,16 @@ std::atomic<uint64_t> g_launches{0};
 }
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
+namespace {
+std::atomic<int> g_fail_launches{0};
+}
+unsigned launch_block() {
+  int n = g_fail_launches.load(std::memory_order_relaxed);
+  while (n > 0 && !g_fail_launches.compare_exchange_weak(n, n - 1, std::memory_order_relaxed)) {
+  }
+  return n > 0 ? 0u : (unsigned)kThreads;
+}
+
 uint32_t grid_cap_for(const void* fn, size_t dyn_smem) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 152;
@@ -333,6 +343,12 @@ extern "C" {
 int sv_abi_version(void) { return SV_ABI_VERSION; }
 
 uint64_t sv_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+int sv_debug_fail_launches(int n) {
+  if (n < 0) return SV_EINVAL;
+  g_fail_launches.store(n, std::memory_order_relaxed);
+  return SV_OK;
+}
 
 int syn_box_muller(const uint32_t* d_words, size_t n_pairs, float* d_z, sv_stream_t stream) {
   if (n_pairs == 0) return SV_OK;

@@ -581,12 +581,12 @@ cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevP
   cp.partials = partials;
   cp.flag = flag;
   switch (dtype) {
-    case SV_F32: cmp_kernel<SV_F32><<<sh.grid, kThreads, 0, st>>>(cp); break;
-    case SV_F16: cmp_kernel<SV_F16><<<sh.grid, kThreads, 0, st>>>(cp); break;
-    case SV_BF16: cmp_kernel<SV_BF16><<<sh.grid, kThreads, 0, st>>>(cp); break;
-    case SV_I32: cmp_kernel<SV_I32><<<sh.grid, kThreads, 0, st>>>(cp); break;
-    case SV_I64: cmp_kernel<SV_I64><<<sh.grid, kThreads, 0, st>>>(cp); break;
-    default: cmp_kernel<SV_U32><<<sh.grid, kThreads, 0, st>>>(cp); break;
+    case SV_F32: cmp_kernel<SV_F32><<<sh.grid, launch_block(), 0, st>>>(cp); break;
+    case SV_F16: cmp_kernel<SV_F16><<<sh.grid, launch_block(), 0, st>>>(cp); break;
+    case SV_BF16: cmp_kernel<SV_BF16><<<sh.grid, launch_block(), 0, st>>>(cp); break;
+    case SV_I32: cmp_kernel<SV_I32><<<sh.grid, launch_block(), 0, st>>>(cp); break;
+    case SV_I64: cmp_kernel<SV_I64><<<sh.grid, launch_block(), 0, st>>>(cp); break;
+    default: cmp_kernel<SV_U32><<<sh.grid, launch_block(), 0, st>>>(cp); break;
   }
   count_launch();
   return cudaGetLastError();
@@ -604,7 +604,7 @@ cudaError_t launch_compare_small(const DevPair* host, const DevPair* dev, int n,
   cp.partials = partials;
   cp.flag = nullptr;
   const unsigned blocks = (unsigned)((n + kThreads / 32 - 1) / (kThreads / 32));
-  cmp_small_kernel<<<blocks, kThreads, 0, st>>>(cp);
+  cmp_small_kernel<<<blocks, launch_block(), 0, st>>>(cp);
   count_launch();
   return cudaGetLastError();
 }
@@ -620,10 +620,10 @@ cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const
   cp.first_group = first_group;
   if (flag) {  // a progressive group: one CTA, stages in order
     if (n > SV_INLINE_ENTRIES || dev) return cudaErrorInvalidValue;
-    combine_stages_kernel<<<1, kThreads, 0, st>>>(cp);
+    combine_stages_kernel<<<1, launch_block(), 0, st>>>(cp);
   } else {
     const uint64_t blocks = ((uint64_t)n * 32 + kThreads - 1) / kThreads;
-    combine_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(cp);
+    combine_kernel<<<(unsigned)blocks, launch_block(), 0, st>>>(cp);
   }
   count_launch();
   return cudaGetLastError();

@@ -574,7 +574,7 @@ cudaError_t launch_generate_group(uint32_t dtype, uint32_t dist, const DevSpec* 
   gp.arena = arena;
   switch (SV_COMBO(dtype, dist)) {
 #define SV_CASE(DT, DIST) \
-  case SV_COMBO(DT, DIST): gen_kernel<DT, DIST><<<sh.grid, kThreads, 0, st>>>(gp); break;
+  case SV_COMBO(DT, DIST): gen_kernel<DT, DIST><<<sh.grid, launch_block(), 0, st>>>(gp); break;
     SV_GEN_COMBOS(SV_CASE)
 #undef SV_CASE
     default: return cudaErrorInvalidValue;
@@ -592,7 +592,7 @@ cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_
   gp.chunk = 0;
   gp.arena = arena;
   const uint64_t blocks = (total_units + kThreads - 1) / kThreads;
-  fixup_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(gp);
+  fixup_kernel<<<(unsigned)blocks, launch_block(), 0, st>>>(gp);
   count_launch();
   return cudaGetLastError();
 }
@@ -602,7 +602,7 @@ static cudaError_t launch_dot(const DotParams& dp, uint64_t tiles, cudaStream_t 
   const void* fn = reinterpret_cast<const void*>(dot_kernel<DT, A16>);
   const uint32_t cap = grid_cap_for(fn, kDotSmem);
   const unsigned grid = (unsigned)std::min<uint64_t>(tiles, cap);
-  dot_kernel<DT, A16><<<grid, kThreads, kDotSmem, st>>>(dp);
+  dot_kernel<DT, A16><<<grid, launch_block(), kDotSmem, st>>>(dp);
   count_launch();
   return cudaGetLastError();
 }
@@ -611,7 +611,7 @@ cudaError_t launch_box_muller(const uint32_t* words, uint64_t n_pairs, float* z,
   if (n_pairs == 0) return cudaSuccess;
   const void* fn = reinterpret_cast<const void*>(box_muller_kernel);
   const uint64_t blocks = std::min<uint64_t>((n_pairs + kThreads - 1) / kThreads, grid_cap_for(fn));
-  box_muller_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(reinterpret_cast<const uint2*>(words), n_pairs,
+  box_muller_kernel<<<(unsigned)blocks, launch_block(), 0, st>>>(reinterpret_cast<const uint2*>(words), n_pairs,
                                                             reinterpret_cast<float2*>(z));
   count_launch();
   return cudaGetLastError();

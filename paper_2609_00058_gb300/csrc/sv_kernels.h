@@ -82,6 +82,10 @@ LaunchShape shape_for(uint64_t units, uint64_t tiles, uint32_t cap, uint64_t ali
 uint32_t grid_cap_for(const void* kernel, size_t dyn_smem = 0);
 // one more kernel launched by this library (the sv_kernel_launches counter)
 void count_launch();
+// the block size of every launch: kThreads, or 0 (an invalid configuration,
+// so the launch fails and no kernel runs) while sv_debug_fail_launches has
+// failures pending
+unsigned launch_block();
 
 SV_HD inline uint64_t cmp_tiles(const vc_pair& p) {
   const uint64_t sz = p.dtype == SV_I64 ? 8 : ((p.dtype == SV_F16 || p.dtype == SV_BF16) ? 2 : 4);

@@ -195,3 +195,9 @@ def test_box_muller_entry_validates_before_any_launch():
     assert lib.syn_box_muller(0x1004, 4, 0x2000, None) == -2       # 4-byte aligned words
     assert lib.syn_box_muller(0x1000, 4, 0x2004, None) == -2       # 4-byte aligned output
     assert lib.syn_box_muller(0x1000, (1 << 39) + 1, 0x2000, None) == -3
+
+
+def test_failure_hook_arguments():
+    lib = sv.lib()
+    assert lib.sv_debug_fail_launches(-1) == -1
+    assert lib.sv_debug_fail_launches(0) == 0
