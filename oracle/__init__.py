@@ -17,6 +17,7 @@ import numpy as np
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 SRC = os.path.join(HERE, "oracle.c")
+SRCS = [SRC, os.path.join(HERE, "convert.c")]
 HDR = os.path.join(HERE, "oracle.h")
 LIB = os.path.join(HERE, "_build", "liboracle.so")
 CFLAGS = ["-O2", "-std=c11", "-Wall", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
@@ -29,6 +30,9 @@ SPECIALS = {"nan": 1, "pinf": 2, "ninf": 4, "denorm": 8, "zero": 16, "imin": 32,
 PERTS = {"none": 0, "rate_add_pm": 1, "rel_noise": 2, "count_set": 3, "count_add": 4, "swap_pairs": 5}
 PURPOSES = {"value": 0, "special_sel": 1, "special_kind": 2, "pert_sel": 3, "pert_val": 4, "index": 5,
             "perm": 6, "noise": 7}
+# element types of test-data files: the six array types and six more
+IO_DTYPES = dict(DTYPES, u8=6, i8=7, i16=8, u16=9, u64=10, f64=11)
+IO_DTYPE_BYTES = dict(DTYPE_BYTES, u8=1, i8=1, i16=2, u16=2, u64=8, f64=8)
 ABSENT = (1 << 64) - 1
 STAGE_RUN, STAGE_SKIPPED = 1, 2
 
@@ -36,10 +40,10 @@ STAGE_RUN, STAGE_SKIPPED = 1, 2
 def build(force: bool = False) -> str:
     """Compile liboracle.so with gcc (seconds)."""
     os.makedirs(os.path.dirname(LIB), exist_ok=True)
-    newest = max(os.path.getmtime(SRC), os.path.getmtime(HDR))
+    newest = max(os.path.getmtime(f) for f in SRCS + [HDR])
     if force or not os.path.exists(LIB) or os.path.getmtime(LIB) < newest:
         tmp = LIB + ".%d.tmp" % os.getpid()
-        subprocess.check_call(["gcc", *CFLAGS, "-o", tmp, SRC, "-lm"])
+        subprocess.check_call(["gcc", *CFLAGS, "-o", tmp, *SRCS, "-lm"])
         os.replace(tmp, LIB)
     return LIB
 
@@ -116,6 +120,10 @@ def lib() -> C.CDLL:
         L.or_progressive.argtypes = [C.POINTER(PairC), C.c_int, C.c_void_p, C.c_uint64, C.c_void_p,
                                      C.c_uint64, C.POINTER(Result), C.POINTER(C.c_int32)]
         L.or_progressive.restype = C.c_int
+        L.or_dtype_bytes.argtypes = [C.c_int]
+        L.or_dtype_bytes.restype = C.c_int
+        L.or_convert.argtypes = [C.c_int, C.c_void_p, C.c_uint64, C.c_int, C.c_void_p, u64p]
+        L.or_convert.restype = C.c_int
         _lib = L
     return _lib
 
@@ -281,3 +289,21 @@ def run_workload(wl, arena: np.ndarray = None):
         res, ff = progressive(wl.pairs, arena, arena)
         return arena, res, ff
     return arena, compare(wl.pairs, arena, arena), None
+
+
+def convert(src: np.ndarray, src_dtype: str, dst_dtype: str) -> Tuple[np.ndarray, int]:
+    """Dtype-correct value conversion of `src` (its bytes are read as
+    `src_dtype` elements): returns (destination bytes as uint8, number of
+    clamped / overflowed elements).  Raises ValueError for a refused pair
+    (float to integer)."""
+    raw = np.ascontiguousarray(src).view(np.uint8).reshape(-1)
+    sb, db = IO_DTYPE_BYTES[src_dtype], IO_DTYPE_BYTES[dst_dtype]
+    assert raw.size % sb == 0
+    n = raw.size // sb
+    out = np.zeros(n * db, np.uint8)
+    bad = C.c_uint64(0)
+    rc = lib().or_convert(IO_DTYPES[src_dtype], raw.ctypes.data, n, IO_DTYPES[dst_dtype], out.ctypes.data,
+                          C.byref(bad))
+    if rc != 0:
+        raise ValueError("conversion %s -> %s refused" % (src_dtype, dst_dtype))
+    return out, bad.value

@@ -138,6 +138,25 @@ int or_compare(const or_pair* pairs, int n_pairs, const uint8_t* cand, uint64_t 
 int or_progressive(const or_pair* stages, int n_stages, const uint8_t* cand, uint64_t cand_bytes,
                    const uint8_t* ref, uint64_t ref_bytes, or_result* out, int32_t* first_failed);
 
+/* ---- value conversion of test data (convert.c) ----
+ * The scaffold's helpers read the prepared test inputs and write the
+ * outputs (Sec. 4.1.2); loading data of one element type as another (every
+ * file read as float) is the loader defect behind 31.4% of the false
+ * positives analysed in Sec. 5.2.3.  A dtype-correct load converts VALUES:
+ *   - same type: the bytes, unchanged (NaN payloads included);
+ *   - integer -> integer: the value; out of the target's range it is clamped
+ *     to the nearest limit and counted in *n_bad;
+ *   - any -> float: the value rounded once to nearest, ties to even, in the
+ *     target format (subnormals kept, no flush to zero); a finite value that
+ *     rounds beyond the largest finite value becomes +-Inf and is counted in
+ *     *n_bad; +-Inf stay; every NaN becomes the target's canonical quiet NaN
+ *     (positive, top fraction bit only); -0 stays -0;
+ *   - float -> integer: refused (-1, nothing written): no silent truncation.
+ * Element types: the six array types above plus the file-only types below. */
+enum { OR_U8 = 6, OR_I8 = 7, OR_I16 = 8, OR_U16 = 9, OR_U64 = 10, OR_F64 = 11 };
+int or_dtype_bytes(int dtype); /* 0 for an unknown type */
+int or_convert(int src_dtype, const void* src, uint64_t n, int dst_dtype, void* dst, uint64_t* n_bad);
+
 #ifdef __cplusplus
 }
 #endif
