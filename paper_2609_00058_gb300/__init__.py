@@ -35,7 +35,14 @@ EQUAL_NAN = 1
 STAGE_RUN, STAGE_SKIPPED = 1, 2
 NO_OUTPUT = (1 << 64) - 1
 INLINE_ENTRIES = 8
-STATUS = {0: "SV_OK", -1: "SV_EINVAL", -2: "SV_EALIGN", -3: "SV_ERANGE", -4: "SV_EWORKSPACE", -5: "SV_ECUDA"}
+STATUS = {0: "SV_OK", -1: "SV_EINVAL", -2: "SV_EALIGN", -3: "SV_ERANGE", -4: "SV_EWORKSPACE", -5: "SV_ECUDA",
+          -6: "SV_EIO", -7: "SV_EFORMAT", -8: "SV_ELOSSY"}
+# element types of test-data files and buffers (include/sv_io.h)
+IO_DTYPES = dict(DTYPES, u8=6, i8=7, i16=8, u16=9, u64=10, f64=11)
+IO_DTYPE_BYTES = dict(DTYPE_BYTES, u8=1, i8=1, i16=2, u16=2, u64=8, f64=8)
+IO_DTYPE_NAMES = {v: k for k, v in IO_DTYPES.items()}
+IO_RAW, IO_STRICT = 1, 2
+TENSOR_MAX_DIMS = 8
 
 
 # ---------------------------------------------------------------------------
@@ -117,7 +124,14 @@ class vc_result(C.Structure):
                 ("state", C.c_uint32)]
 
 
+class sv_tensor_header(C.Structure):
+    _fields_ = [("magic", C.c_uint32), ("header_bytes", C.c_uint32), ("dtype", C.c_uint32), ("ndim", C.c_uint32),
+                ("shape", C.c_uint64 * TENSOR_MAX_DIMS), ("n", C.c_uint64), ("data_bytes", C.c_uint64),
+                ("reserved", C.c_uint64 * 4)]
+
+
 assert C.sizeof(syn_spec) == 224 and C.sizeof(vc_pair) == 48 and C.sizeof(vc_result) == 80
+assert C.sizeof(sv_tensor_header) == 128
 RESULT_BYTES = C.sizeof(vc_result)
 
 # every function the header declares: (name, restype, argtypes)
@@ -137,6 +151,15 @@ EXPORTS = [
     ("sv_kernel_launches", C.c_uint64, []),
     ("syn_box_muller", C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
     ("sv_debug_fail_launches", C.c_int, [C.c_int]),
+    # include/sv_io.h
+    ("sv_dtype_bytes", C.c_int, [C.c_int]),
+    ("sv_tensor_probe", C.c_int, [C.c_char_p, C.POINTER(sv_tensor_header)]),
+    ("sv_io_workspace_bytes", _SZ, [C.c_int, C.c_int, C.c_uint64]),
+    ("sv_read_tensor", C.c_int, [C.c_char_p, C.c_uint32, C.c_int, C.c_uint64, C.c_int, _VP, _SZ, _VP, _SZ, _VP,
+                                 C.POINTER(sv_tensor_header), C.POINTER(C.c_uint64)]),
+    ("sv_write_tensor", C.c_int, [C.c_char_p, C.c_uint32, C.c_int, C.POINTER(C.c_uint64), C.c_int, _VP, _SZ, _VP]),
+    ("sv_convert", C.c_int, [C.c_int, _VP, C.c_uint64, C.c_int, _VP, _VP, _VP]),
+    ("sv_debug_io_chunk_bytes", C.c_int, [_SZ]),
 ]
 
 _lib = None
@@ -315,3 +338,104 @@ def check_specs(specs, arena_bytes: int) -> int:
 def check_pairs(pairs, cand_bytes: int, ref_bytes: int) -> int:
     tab = PairTable(pairs)
     return lib().sv_check_pairs(tab.arr, tab.n, cand_bytes, ref_bytes)
+
+
+# ---------------------------------------------------------------------------
+# test-data I/O (include/sv_io.h)
+# ---------------------------------------------------------------------------
+def _torch_dtype(name: str):
+    import torch
+    return {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16, "f64": torch.float64,
+            "i32": torch.int32, "i64": torch.int64, "i16": torch.int16, "i8": torch.int8, "u8": torch.uint8,
+            "u16": torch.uint16, "u32": torch.uint32, "u64": torch.uint64}[name]
+
+
+def _header_dict(h: sv_tensor_header) -> dict:
+    return {"dtype": IO_DTYPE_NAMES.get(h.dtype, h.dtype), "ndim": h.ndim, "shape": tuple(h.shape[: h.ndim]),
+            "n": h.n, "data_bytes": h.data_bytes}
+
+
+def _path(path) -> bytes:
+    return os.fsencode(os.fspath(path))
+
+
+def tensor_probe(path) -> dict:
+    """sv_tensor_probe: the checked header of a tensor file."""
+    h = sv_tensor_header()
+    _ok(lib().sv_tensor_probe(_path(path), C.byref(h)), "sv_tensor_probe")
+    return _header_dict(h)
+
+
+def read_tensor(path, dtype: Optional[str] = None, out=None, *, file_dtype: Optional[str] = None,
+                n: Optional[int] = None, raw: bool = False, strict: bool = False, lossy_ok: bool = False,
+                device=None, workspace=None, stream=None):
+    """sv_read_tensor: load a test-data file into device memory, converting
+    values to `dtype` (default: the file's type).  Returns (tensor, header,
+    lost): the tensor has the file's shape when `out` is not given, else it is
+    `out` (a CUDA tensor whose bytes receive the data).  Raises on every error,
+    and on lost values (clamped or overflowed) unless lossy_ok."""
+    import torch
+    flags = (IO_RAW if raw else 0) | (IO_STRICT if strict else 0)
+    if raw:
+        if file_dtype is None:
+            raise ValueError("a headerless file needs file_dtype")
+        shape, src = None, file_dtype
+        if n is None:
+            n_file = os.path.getsize(path) // IO_DTYPE_BYTES[file_dtype]
+        else:
+            n_file = n
+    else:
+        info = tensor_probe(path)
+        shape, src, n_file = info["shape"], info["dtype"], info["n"]
+    dst = dtype or src
+    if out is not None:
+        dev = out.device
+    else:
+        dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+    if out is None:
+        buf = torch.empty(max(n_file, 1) * IO_DTYPE_BYTES[dst], dtype=torch.uint8, device=dev)
+    else:
+        buf = out
+    ws = _workspace(lib().sv_io_workspace_bytes(IO_DTYPES[src], IO_DTYPES[dst], n_file), dev, workspace)
+    h = sv_tensor_header()
+    lost = C.c_uint64(0)
+    rc = lib().sv_read_tensor(_path(path), flags, -1 if file_dtype is None else IO_DTYPES[file_dtype],
+                              n or 0, IO_DTYPES[dst], buf.data_ptr(), _nbytes(buf), ws[0], ws[1] if ws[0] else 0,
+                              _stream_ptr(stream), C.byref(h), C.byref(lost))
+    if rc != -8 or not lossy_ok:
+        _ok(rc, "sv_read_tensor")
+    hd = _header_dict(h)
+    if out is None:
+        t = buf[: hd["n"] * IO_DTYPE_BYTES[dst]].view(_torch_dtype(dst))
+        out = t.reshape(hd["shape"]) if not raw else t
+    return out, hd, lost.value
+
+
+def write_tensor(path, src, dtype: Optional[str] = None, shape: Optional[Sequence[int]] = None, raw: bool = False,
+                 stream=None) -> None:
+    """sv_write_tensor: write a CUDA tensor's bytes to a tensor file (header
+    with `dtype` and `shape`, default: the tensor's own)."""
+    if dtype is None:
+        names = {_torch_dtype(k): k for k in IO_DTYPES}
+        dtype = names[src.dtype]
+    if shape is None:  # the tensor's own shape, or its bytes as a vector of `dtype`
+        shape = tuple(src.shape) if src.dtype == _torch_dtype(dtype) else (_nbytes(src) // IO_DTYPE_BYTES[dtype],)
+    arr = (C.c_uint64 * max(len(shape), 1))(*shape)
+    rc = lib().sv_write_tensor(_path(path), IO_RAW if raw else 0, IO_DTYPES[dtype], arr, len(shape), src.data_ptr(),
+                               _nbytes(src), _stream_ptr(stream))
+    _ok(rc, "sv_write_tensor")
+
+
+def convert(src, src_dtype: str, dst_dtype: str, n: Optional[int] = None, out=None, lost=None, stream=None):
+    """sv_convert: device-to-device value conversion; returns (out, lost),
+    `lost` a device uint64 counter (added to, not reset, when given)."""
+    import torch
+    if n is None:
+        n = _nbytes(src) // IO_DTYPE_BYTES[src_dtype]
+    if out is None:
+        out = torch.empty(max(n, 1) * IO_DTYPE_BYTES[dst_dtype], dtype=torch.uint8, device=src.device)
+    if lost is None:
+        lost = torch.zeros(1, dtype=torch.int64, device=src.device)
+    _ok(lib().sv_convert(IO_DTYPES[src_dtype], src.data_ptr(), n, IO_DTYPES[dst_dtype], out.data_ptr(),
+                         lost.data_ptr(), _stream_ptr(stream)), "sv_convert")
+    return out, lost

@@ -12,6 +12,7 @@
 #include <vector>
 
 #include "sv_device.cuh"
+#include "../../include/sv_io.h"
 #include "sv_kernels.h"
 
 namespace sv {
@@ -366,6 +367,9 @@ const char* sv_strerror(int status) {
     case SV_ERANGE: return "data beyond its buffer, or a size beyond the library limits";
     case SV_EWORKSPACE: return "workspace missing, misaligned or too small";
     case SV_ECUDA: return "a CUDA launch or copy failed";
+    case SV_EIO: return "a file could not be opened, read, written or sized";
+    case SV_EFORMAT: return "bad tensor header, or the file's type, count or size is not the one stated";
+    case SV_ELOSSY: return "data loaded, but values were clamped or overflowed by the type conversion";
     default: return "unknown status";
   }
 }

@@ -140,4 +140,11 @@ cudaError_t launch_compare_small(const DevPair* host, const DevPair* dev, int n,
 cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const Partial* partials,
                            vc_result* results, int32_t* flag, int first_group, cudaStream_t st);
 
+// ---- value conversion of test data (convert.cu) ----
+// n elements of type s at src become n elements of type d at dst (16-byte
+// aligned, s != d, not float -> integer); clamped or overflowed values are
+// added to *lost
+cudaError_t launch_convert(int s, int d, const void* src, void* dst, uint64_t n, unsigned long long* lost,
+                           cudaStream_t st);
+
 }  // namespace sv
