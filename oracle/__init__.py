@@ -67,6 +67,13 @@ class PairC(C.Structure):
                 ("ref_offset", C.c_uint64), ("atol", C.c_double), ("rtol", C.c_double)]
 
 
+class TilesC(C.Structure):
+    _fields_ = [("dtype", C.c_uint32), ("flags", C.c_uint32), ("rows", C.c_uint64), ("cols", C.c_uint64),
+                ("cand_offset", C.c_uint64), ("ref_offset", C.c_uint64), ("cand_pitch", C.c_uint64),
+                ("ref_pitch", C.c_uint64), ("tile_rows", C.c_uint64), ("tile_cols", C.c_uint64),
+                ("atol", C.c_double), ("rtol", C.c_double)]
+
+
 class Result(C.Structure):
     _fields_ = [("mismatches", C.c_uint64), ("nan_disagree", C.c_uint64), ("inf_disagree", C.c_uint64),
                 ("n_finite", C.c_uint64), ("first_mismatch", C.c_int64), ("max_abs_u64", C.c_uint64),
@@ -120,6 +127,9 @@ def lib() -> C.CDLL:
         L.or_progressive.argtypes = [C.POINTER(PairC), C.c_int, C.c_void_p, C.c_uint64, C.c_void_p,
                                      C.c_uint64, C.POINTER(Result), C.POINTER(C.c_int32)]
         L.or_progressive.restype = C.c_int
+        L.or_compare_tiles.argtypes = [C.POINTER(TilesC), C.c_void_p, C.c_uint64, C.c_void_p, C.c_uint64,
+                                       C.POINTER(Result)]
+        L.or_compare_tiles.restype = C.c_int
         L.or_dtype_bytes.argtypes = [C.c_int]
         L.or_dtype_bytes.restype = C.c_int
         L.or_convert.argtypes = [C.c_int, C.c_void_p, C.c_uint64, C.c_int, C.c_void_p, u64p]
@@ -307,3 +317,21 @@ def convert(src: np.ndarray, src_dtype: str, dst_dtype: str) -> Tuple[np.ndarray
     if rc != 0:
         raise ValueError("conversion %s -> %s refused" % (src_dtype, dst_dtype))
     return out, bad.value
+
+
+def tile_grid(t) -> Tuple[int, int]:
+    return (-(-t.rows // t.tile_rows), -(-t.cols // t.tile_cols))
+
+
+def compare_tiles(t, cand: np.ndarray, ref: np.ndarray) -> List[dict]:
+    """Tile-by-tile verdicts of a shaped output `t` (any object with the
+    fields of workloads.Tiles), row-major over the tile grid."""
+    tr, tc = tile_grid(t)
+    n = tr * tc
+    out = (Result * max(n, 1))()
+    c = TilesC(DTYPES[t.dtype], 1 if t.equal_nan else 0, t.rows, t.cols, t.cand_offset, t.ref_offset,
+               t.cand_pitch, t.ref_pitch, t.tile_rows, t.tile_cols, t.atol, t.rtol)
+    rc = lib().or_compare_tiles(C.byref(c), cand.ctypes.data, cand.nbytes, ref.ctypes.data, ref.nbytes, out)
+    if rc != 0:
+        raise ValueError("invalid tiles")
+    return [result_dict(out[i]) for i in range(n)]

@@ -14,6 +14,7 @@
 #include "oracle.h"
 
 #include <math.h>
+#include <stdlib.h>
 #include <string.h>
 
 /* ------------------------------------------------------------------------ */
@@ -675,6 +676,48 @@ int or_compare(const or_pair* pairs, int n_pairs, const uint8_t* cand, uint64_t 
   for (int i = 0; i < n_pairs; ++i)
     if (check_pair(&pairs[i], cand_bytes, ref_bytes) != 0) return -1;
   for (int i = 0; i < n_pairs; ++i) compare_one(&pairs[i], cand, ref, &out[i]);
+  return 0;
+}
+
+/* shaped outputs: a rows x cols output (row-major, row pitches in elements) */
+/* compared tile by tile.  Each tile's elements are gathered in row-major   */
+/* order into dense buffers and compared as one segment by the rule above;  */
+/* its first mismatch is reported as the output-wide index row * cols + col.*/
+int or_compare_tiles(const or_tiles* t, const uint8_t* cand, uint64_t cand_bytes, const uint8_t* ref,
+                     uint64_t ref_bytes, or_result* out) {
+  uint64_t sz = elem_bytes(t->dtype);
+  if (sz == 0 || t->tile_rows == 0 || t->tile_cols == 0) return -1;
+  if (t->cand_pitch < t->cols || t->ref_pitch < t->cols) return -1;
+  if (is_float_dtype(t->dtype) && !(t->atol >= 0.0 && t->rtol >= 0.0)) return -1;
+  if (t->rows && t->cols) { /* the last element of each operand lies inside its buffer */
+    uint64_t xe = t->cand_offset + ((t->rows - 1) * t->cand_pitch + t->cols) * sz;
+    uint64_t ye = t->ref_offset + ((t->rows - 1) * t->ref_pitch + t->cols) * sz;
+    if (xe > cand_bytes || ye > ref_bytes) return -1;
+  }
+  uint64_t ntr = (t->rows + t->tile_rows - 1) / t->tile_rows, ntc = (t->cols + t->tile_cols - 1) / t->tile_cols;
+  uint8_t* xt = (uint8_t*)malloc(t->tile_rows * t->tile_cols * sz + 1);
+  uint8_t* yt = (uint8_t*)malloc(t->tile_rows * t->tile_cols * sz + 1);
+  if (!xt || !yt) { free(xt); free(yt); return -1; }
+  for (uint64_t i = 0; i < ntr; ++i) {
+    for (uint64_t j = 0; j < ntc; ++j) {
+      uint64_t r0 = i * t->tile_rows, r1 = r0 + t->tile_rows < t->rows ? r0 + t->tile_rows : t->rows;
+      uint64_t c0 = j * t->tile_cols, c1 = c0 + t->tile_cols < t->cols ? c0 + t->tile_cols : t->cols;
+      uint64_t w = c1 - c0, k = 0;
+      for (uint64_t r = r0; r < r1; ++r, k += w) {
+        memcpy(xt + k * sz, cand + t->cand_offset + (r * t->cand_pitch + c0) * sz, w * sz);
+        memcpy(yt + k * sz, ref + t->ref_offset + (r * t->ref_pitch + c0) * sz, w * sz);
+      }
+      or_pair p = {t->dtype, t->flags, (r1 - r0) * w, 0, 0, t->atol, t->rtol};
+      or_result* r = &out[i * ntc + j];
+      compare_one(&p, xt, yt, r);
+      if (r->first_mismatch >= 0) {
+        uint64_t f = (uint64_t)r->first_mismatch;
+        r->first_mismatch = (int64_t)((r0 + f / w) * t->cols + c0 + f % w);
+      }
+    }
+  }
+  free(xt);
+  free(yt);
   return 0;
 }
 

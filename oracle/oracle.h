@@ -138,6 +138,24 @@ int or_compare(const or_pair* pairs, int n_pairs, const uint8_t* cand, uint64_t 
 int or_progressive(const or_pair* stages, int n_stages, const uint8_t* cand, uint64_t cand_bytes,
                    const uint8_t* ref, uint64_t ref_bytes, or_result* out, int32_t* first_failed);
 
+/* ---- shaped outputs (Sec. 4.1.1: the manifest gives each output's shape) ----
+ * A rows x cols output, row-major, with a row pitch (elements between row
+ * starts, >= cols) per operand, cut into tiles of tile_rows x tile_cols (the
+ * last tile row / column may be smaller).  out[i * tiles_per_row + j] is the
+ * verdict of tile (i, j) by the rule of or_compare over its elements in
+ * row-major order; first_mismatch is the output-wide index row * cols + col.
+ * Returns -1 (nothing written) for an invalid description. */
+typedef struct {
+  uint32_t dtype, flags;
+  uint64_t rows, cols;
+  uint64_t cand_offset, ref_offset;
+  uint64_t cand_pitch, ref_pitch;
+  uint64_t tile_rows, tile_cols;
+  double atol, rtol;
+} or_tiles;
+int or_compare_tiles(const or_tiles* t, const uint8_t* cand, uint64_t cand_bytes, const uint8_t* ref,
+                     uint64_t ref_bytes, or_result* out);
+
 /* ---- value conversion of test data (convert.c) ----
  * The scaffold's helpers read the prepared test inputs and write the
  * outputs (Sec. 4.1.2); loading data of one element type as another (every

@@ -81,6 +81,30 @@ class Pair:
     equal_nan: bool = True
 
 
+@dataclass
+class Tiles:
+    """A 2-D output (rows x cols elements, row-major) compared tile by tile;
+    each operand has its own row pitch (elements between row starts).  Zero
+    pitches and a zero tile_cols mean cols."""
+    dtype: str
+    rows: int
+    cols: int
+    cand_offset: int
+    ref_offset: int
+    cand_pitch: int = 0
+    ref_pitch: int = 0
+    tile_rows: int = 1
+    tile_cols: int = 0
+    atol: float = 0.0
+    rtol: float = 0.0
+    equal_nan: bool = True
+
+    def __post_init__(self):
+        self.cand_pitch = self.cand_pitch or self.cols
+        self.ref_pitch = self.ref_pitch or self.cols
+        self.tile_cols = self.tile_cols or self.cols
+
+
 class Arena:
     """Bump allocator for byte offsets inside one arena."""
 
