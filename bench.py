@@ -13,7 +13,11 @@ the public API with the synthesized test data delivered to pinned host
 memory and the verdicts read back every step.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--workload ladder|fp32_pair|segmented|dotlike_bf16|perm_i64]
+                  [--workload ladder|fp32_pair|segmented|dotlike_bf16|perm_i64|tensor_io]
+
+--workload tensor_io measures the test-data I/O path instead (sv_read_tensor
+of a 1 GiB uint8 tensor file into fp32, the conversion kernel alone, the
+pinned copy rate and sv_write_tensor) and prints its own JSON line.
 
 Under torchrun (N > 1) every rank runs an independent replica on its own
 GPU (the path needs no exchange at this size); the time is the max over ranks.
@@ -233,6 +237,8 @@ def reference_arm(args, rank, world):
         return
     import oracle
     oracle.build()
+    if args.workload == "tensor_io":
+        return io_reference_arm(args)
     wl, sample = oracle_sample(args.workload)
     for _ in range(args.warmup):
         run_oracle_once(wl)
@@ -250,6 +256,39 @@ def reference_arm(args, rank, world):
             "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def io_reference_arm(args):
+    """The oracle's load of test data: a 16 MiB uint8 file read by numpy and
+    converted to fp32 by the oracle, per step."""
+    import shutil
+    import tempfile
+
+    import oracle
+    host = np.random.default_rng(0).integers(0, 256, size=16 << 20, dtype=np.uint8)
+    tmp = tempfile.mkdtemp(prefix="svio_")
+    try:
+        p = os.path.join(tmp, "s.bin")
+        host.tofile(p)
+        for _ in range(args.warmup):
+            oracle.convert(np.fromfile(p, np.uint8), "u8", "f32")
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            oracle.convert(np.fromfile(p, np.uint8), "u8", "f32")
+        tot = time.perf_counter() - t0
+    finally:
+        shutil.rmtree(tmp, ignore_errors=True)
+    value = host.size * args.steps / tot / 1e9
+    sample = "16 MiB uint8 file read by numpy, converted to fp32 by the oracle (single thread)"
+    print(json.dumps({"impl": "reference", "metric": IO_METRIC, "value": value, "unit": "GB/s", "n_gpus": args.gpus,
+                      "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+                      "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8->f32",
+                      "data": "synthetic (uniform random bytes)",
+                      "config": {"workload": "1 GiB uint8 tensor file loaded as fp32", "sample": sample},
+                      "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                       "sample": sample},
+                      "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}),
+          flush=True)
 
 
 # ---------------------------------------------------------------------------
@@ -484,6 +523,152 @@ def ours_arm(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+# ---------------------------------------------------------------------------
+# the test-data I/O path (include/sv_io.h)
+# ---------------------------------------------------------------------------
+IO_METRIC = "test-data load GB/s (file bytes into HBM, values converted) on 1 GB300"
+IO_FILE_ELEMS = 1 << 30  # uint8 elements of the timed file (1 GiB), loaded as fp32 (4 GiB)
+IO_CONVERSIONS = [("u8", "f32"), ("f32", "bf16"), ("i32", "f32"), ("f64", "f32"), ("f32", "f64"), ("i64", "f32"),
+                  ("f64", "bf16"), ("i32", "f64"), ("u16", "f16")]
+
+
+def io_arm(args, rank, world):
+    """One step = sv_read_tensor of a 1 GiB uint8 tensor file (page cache warm)
+    into an fp32 buffer: host threads read the file into pinned chunks, the
+    chunks cross to the GPU and the GPU converts each one.  Also measured: the
+    conversion kernel alone (device to device, HBM roofline), the pinned
+    host-to-device copy rate (the link's ceiling for the file path) and
+    sv_write_tensor of the same bytes."""
+    import shutil
+    import tempfile
+
+    import torch
+
+    import oracle
+    import paper_2609_00058_gb300 as sv
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    n = IO_FILE_ELEMS
+    src = torch.randint(0, 256, (n,), dtype=torch.uint8, device=dev)
+    out = torch.empty(4 * n, dtype=torch.uint8, device=dev)
+    ws = torch.empty(sv.lib().sv_io_workspace_bytes(sv.IO_DTYPES["u8"], sv.IO_DTYPES["f32"], n),
+                     dtype=torch.uint8, device=dev)
+    tmp = tempfile.mkdtemp(prefix="svio_")
+    path = os.path.join(tmp, "input.svt")
+    try:
+        t0 = time.perf_counter()
+        sv.write_tensor(path, src, dtype="u8", shape=(n,))
+        write_s = time.perf_counter() - t0
+        for _ in range(max(args.warmup, 3)):
+            sv.read_tensor(path, dtype="f32", out=out, workspace=ws)
+        torch.cuda.synchronize()
+        barrier(world)
+        sampler = ClockSampler(dev)
+        sampler.start()
+        time.sleep(0.05)
+        launches0 = sv.lib().sv_kernel_launches()
+        times = []
+        t_host0 = time.perf_counter()
+        for _ in range(args.steps):
+            t0 = time.perf_counter()
+            sv.read_tensor(path, dtype="f32", out=out, workspace=ws)  # returns with the data in place
+            times.append(time.perf_counter() - t0)
+        t_host1 = time.perf_counter()
+        launches = sv.lib().sv_kernel_launches() - launches0
+        clocks = sampler.stop(t_host0, t_host1)
+        total_s = max_over_ranks(sum(times), world)
+        ok = bool(torch.equal(out.view(torch.float32)[:: 1 << 16], src[:: 1 << 16].float()))
+        t0 = time.perf_counter()
+        for _ in range(3):
+            sv.write_tensor(path, src, dtype="u8", shape=(n,))
+        write_s = min(write_s, (time.perf_counter() - t0) / 3)
+    finally:
+        shutil.rmtree(tmp, ignore_errors=True)
+
+    # the conversion kernel alone, inputs resident (larger than L2)
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    conv = {}
+    lost = torch.zeros(1, dtype=torch.int64, device=dev)
+    for s_t, d_t in IO_CONVERSIONS:
+        m = (1 << 30) // sv.IO_DTYPE_BYTES[s_t]  # 1 GiB of source
+        a = torch.randint(0, 256, (m * sv.IO_DTYPE_BYTES[s_t],), dtype=torch.uint8, device=dev)
+        if s_t in ("f32", "f64"):  # finite float test values rather than random encodings
+            a = (torch.randn(m, device=dev, dtype=torch.float64 if s_t == "f64" else torch.float32)
+                 * 100).view(torch.uint8)
+        elif s_t in ("i32", "i64"):  # integers of every magnitude
+            a = torch.randint(-2 ** 31, 2 ** 31, (m,), device=dev, dtype=torch.int64)
+            a = (a if s_t == "i64" else a.to(torch.int32)).view(torch.uint8)
+        b = torch.empty(m * sv.IO_DTYPE_BYTES[d_t], dtype=torch.uint8, device=dev)
+        for _ in range(3):
+            sv.convert(a, s_t, d_t, n=m, out=b, lost=lost)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(5, min(args.steps, 20))
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            sv.convert(a, s_t, d_t, n=m, out=b, lost=lost)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        nbytes = m * (sv.IO_DTYPE_BYTES[s_t] + sv.IO_DTYPE_BYTES[d_t])
+        conv["%s->%s" % (s_t, d_t)] = {"ms": ms, "bytes": nbytes, "gbs": nbytes / (ms * 1e-3) / 1e9,
+                                       "frac_of_hbm": nbytes / (ms * 1e-3) / 1e9 / hbm}
+        del a, b
+    # the link: pinned host -> device copy of 1 GiB
+    pinned = torch.empty(1 << 30, dtype=torch.uint8, pin_memory=True)
+    for _ in range(2):
+        out[: 1 << 30].copy_(pinned, non_blocking=True)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(5):
+        out[: 1 << 30].copy_(pinned, non_blocking=True)
+    torch.cuda.synchronize()
+    link_gbs = 5 * (1 << 30) / (time.perf_counter() - t0) / 1e9
+    if rank != 0:
+        return
+    value = world * n * args.steps / total_s / 1e9
+    main_conv = conv["u8->f32"]
+    line = {
+        "metric": IO_METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * total_s / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u8->f32", "data": "synthetic (uniform random bytes)",
+        "config": {"workload": "1 GiB uint8 tensor file loaded as fp32 (sv_read_tensor, page cache warm)",
+                   "file_bytes": n + 128, "loaded_bytes": 4 * n, "chunk_bytes": 32 << 20,
+                   "host_threads": os.cpu_count(), "l2": "1 GiB source, 4 GiB destination: larger than L2",
+                   "values_checked": ok, "parallelism": "replicas" if world > 1 else "single GPU"},
+        "roofline": {"bound": "hbm", "kernel": "cvt_kernel<u8, f32> (sv_convert, device to device)",
+                     "achieved": main_conv["gbs"], "peak": hbm, "unit": "GB/s", "frac": main_conv["frac_of_hbm"],
+                     "peak_kind": "%s (%s)" % (peak_kind, "hbm_gbs"), "traffic": None},
+        "convert": conv,
+        "link_h2d_gbs": link_gbs, "file_path_frac_of_link": value / world / link_gbs,
+        "write_gbs": n / write_s / 1e9,
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": n, "d2h_bytes_per_step": 0,
+                "what": "the public call itself: file on the host, result in HBM"},
+        "clocks": clocks, "gpu_launches": launches,
+    }
+    if not args.no_cpu_baseline:  # the oracle's conversion after a numpy read of the same bytes
+        host = np.random.default_rng(0).integers(0, 256, size=16 << 20, dtype=np.uint8)
+        tmp = tempfile.mkdtemp(prefix="svio_")
+        try:
+            p = os.path.join(tmp, "s.bin")
+            host.tofile(p)
+            tot, reps = 0.0, 0
+            while reps == 0 or tot < CPU_BASELINE_SECONDS:
+                t0 = time.perf_counter()
+                oracle.convert(np.fromfile(p, np.uint8), "u8", "f32")
+                tot += time.perf_counter() - t0
+                reps += 1
+        finally:
+            shutil.rmtree(tmp, ignore_errors=True)
+        line["cpu_baseline"] = {"value": reps * host.size / tot / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                "sample": "%d x (16 MiB uint8 file read by numpy, converted to fp32 by the oracle), "
+                                          "%.1f s" % (reps, tot)}
+    print(json.dumps(line), flush=True)
+
+
 def barrier(world):
     if world > 1:
         import torch.distributed as dist
@@ -515,7 +700,7 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="ladder", choices=sorted(W.FULL_SIZE))
+    ap.add_argument("--workload", default="ladder", choices=sorted(W.FULL_SIZE) + ["tensor_io"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -535,7 +720,7 @@ def main():
             build()
         barrier(world)
         build()
-        ours_arm(args, rank, world)
+        (io_arm if args.workload == "tensor_io" else ours_arm)(args, rank, world)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()

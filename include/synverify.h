@@ -196,6 +196,31 @@ typedef struct vc_result {
   uint32_t state;          /* SV_STAGE_RUN or SV_STAGE_SKIPPED */
 } vc_result;
 
+/* One shaped output compared tile by tile (CUDA-Harness Sec. 4.1.1: the
+ * manifest gives every output's shape and type; Eq. 1 per element).  A
+ * rows x cols output, row-major; the rows of each operand start cand_pitch /
+ * ref_pitch elements apart (>= cols), so a padded or sub-matrix view works.
+ * Tiles of tile_rows x tile_cols cover it in row-major order; the last tile
+ * row and column may be smaller.  A tile of one row and all columns gives
+ * per-row verdicts; a block tile localises an error to the part of the output
+ * that one block of the kernel under test wrote. */
+typedef struct vc_tiles {
+  uint32_t dtype;        /* SV_F32 ... SV_U32 */
+  uint32_t flags;        /* SV_EQUAL_NAN */
+  uint64_t rows, cols;
+  uint64_t cand_offset;  /* byte offset of element (0, 0), multiple of 16 */
+  uint64_t ref_offset;
+  uint64_t cand_pitch;   /* elements from one row start to the next, >= cols;
+                            pitch * size a multiple of 16 when rows > 1 */
+  uint64_t ref_pitch;
+  uint64_t tile_rows;    /* >= 1 */
+  uint64_t tile_cols;    /* >= 1; tile_cols * size a multiple of 16 when
+                            tile_cols < cols */
+  double atol, rtol;     /* as vc_pair */
+} vc_tiles;
+
+#define SV_MAX_TILES ((1ull << 31) - 1)  /* tiles of one call */
+
 /* ---- workspace sizes (host only; no device needed) ----
  * Bytes of device workspace the matching call needs for these tables, 0 for
  * an invalid table.  The workspace must be 256-byte aligned. */
@@ -206,6 +231,8 @@ size_t sv_progressive_workspace_bytes(const vc_pair* stages, int n_stages);
 /* ---- host-only validation (no CUDA call; usable without a GPU) ---- */
 int sv_check_specs(const syn_spec* specs, int n_specs, size_t arena_bytes);
 int sv_check_pairs(const vc_pair* pairs, int n_pairs, size_t cand_bytes, size_t ref_bytes);
+/* also returns the number of tiles (0 on an error) in *n_tiles when not null */
+int sv_check_tiles(const vc_tiles* tiles, size_t cand_bytes, size_t ref_bytes, uint64_t* n_tiles);
 
 /* syn_generate: test-data synthesis (CUDA-Harness Sec. 4.2.1, "Decoupled Test
  * Data Synthesis": inputs and reference data made by seeded numerical
@@ -241,6 +268,20 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
 int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, size_t cand_bytes,
                        const void* d_ref, size_t ref_bytes, vc_result* d_results, int32_t* d_first_failed,
                        void* d_ws, size_t ws_bytes, sv_stream_t stream);
+
+/* verify_compare_tiles: Eq. 1 over a shaped output, one vc_result per tile
+ * (d_results: ceil(rows / tile_rows) * ceil(cols / tile_cols) records,
+ * row-major over the tile grid).  A tile's statistics are those of
+ * verify_compare over its elements in row-major order, except that
+ * first_mismatch is the output-wide index row * cols + col.  Bytes between
+ * the end of a row and the next row start (the pitch padding) are never read.
+ * One CTA reduces a whole tile (no workspace); the GPU fills up with a few
+ * hundred tiles or more.  rows or cols 0: nothing to do.
+ * Errors: SV_EINVAL (type, flags, tolerance, zero tile extent, pitch < cols,
+ * a tile wider or taller than 2^31 - 1), SV_EALIGN, SV_ERANGE (operand beyond
+ * its buffer, more than SV_MAX_TILES tiles), SV_ECUDA. */
+int verify_compare_tiles(const vc_tiles* tiles, const void* d_cand, size_t cand_bytes, const void* d_ref,
+                         size_t ref_bytes, vc_result* d_results, sv_stream_t stream);
 
 /* verify_compare_noalloc: the verdicts of verify_compare for callers that
  * cannot allocate device memory, for instance code running inside a host

@@ -124,6 +124,13 @@ class vc_result(C.Structure):
                 ("state", C.c_uint32)]
 
 
+class vc_tiles(C.Structure):
+    _fields_ = [("dtype", C.c_uint32), ("flags", C.c_uint32), ("rows", C.c_uint64), ("cols", C.c_uint64),
+                ("cand_offset", C.c_uint64), ("ref_offset", C.c_uint64), ("cand_pitch", C.c_uint64),
+                ("ref_pitch", C.c_uint64), ("tile_rows", C.c_uint64), ("tile_cols", C.c_uint64),
+                ("atol", C.c_double), ("rtol", C.c_double)]
+
+
 class sv_tensor_header(C.Structure):
     _fields_ = [("magic", C.c_uint32), ("header_bytes", C.c_uint32), ("dtype", C.c_uint32), ("ndim", C.c_uint32),
                 ("shape", C.c_uint64 * TENSOR_MAX_DIMS), ("n", C.c_uint64), ("data_bytes", C.c_uint64),
@@ -131,7 +138,7 @@ class sv_tensor_header(C.Structure):
 
 
 assert C.sizeof(syn_spec) == 224 and C.sizeof(vc_pair) == 48 and C.sizeof(vc_result) == 80
-assert C.sizeof(sv_tensor_header) == 128
+assert C.sizeof(sv_tensor_header) == 128 and C.sizeof(vc_tiles) == 88
 RESULT_BYTES = C.sizeof(vc_result)
 
 # every function the header declares: (name, restype, argtypes)
@@ -151,6 +158,8 @@ EXPORTS = [
     ("sv_kernel_launches", C.c_uint64, []),
     ("syn_box_muller", C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
     ("sv_debug_fail_launches", C.c_int, [C.c_int]),
+    ("sv_check_tiles", C.c_int, [C.POINTER(vc_tiles), _SZ, _SZ, C.POINTER(C.c_uint64)]),
+    ("verify_compare_tiles", C.c_int, [C.POINTER(vc_tiles), _VP, _SZ, _VP, _SZ, _VP, _VP]),
     # include/sv_io.h
     ("sv_dtype_bytes", C.c_int, [C.c_int]),
     ("sv_tensor_probe", C.c_int, [C.c_char_p, C.POINTER(sv_tensor_header)]),
@@ -305,6 +314,32 @@ def progressive(stages, cand, ref, results=None, first_failed=None, workspace=No
                                   _stream_ptr(stream))
     _ok(rc, "verify_progressive")
     return results, first_failed
+
+
+def to_c_tiles(t) -> vc_tiles:
+    """A shaped output (any object with the fields of workloads.Tiles)."""
+    return vc_tiles(DTYPES[t.dtype], EQUAL_NAN if t.equal_nan else 0, t.rows, t.cols, t.cand_offset, t.ref_offset,
+                    t.cand_pitch or t.cols, t.ref_pitch or t.cols, t.tile_rows, t.tile_cols or t.cols, t.atol, t.rtol)
+
+
+def tile_count(t, cand_bytes: int = 1 << 62, ref_bytes: int = 1 << 62) -> int:
+    """sv_check_tiles: the number of tiles (raises on an invalid description)."""
+    n = C.c_uint64(0)
+    _ok(lib().sv_check_tiles(C.byref(to_c_tiles(t)), cand_bytes, ref_bytes, C.byref(n)), "sv_check_tiles")
+    return n.value
+
+
+def compare_tiles(tiles, cand, ref, results=None, stream=None):
+    """verify_compare_tiles; returns the device results tensor (uint8, one
+    80-byte vc_result per tile, row-major over the tile grid)."""
+    import torch
+    c = to_c_tiles(tiles)
+    n = tile_count(tiles, _nbytes(cand), _nbytes(ref))
+    if results is None:
+        results = torch.empty(max(n, 1) * RESULT_BYTES, dtype=torch.uint8, device=cand.device)
+    _ok(lib().verify_compare_tiles(C.byref(c), cand.data_ptr(), _nbytes(cand), ref.data_ptr(), _nbytes(ref),
+                                   results.data_ptr(), _stream_ptr(stream)), "verify_compare_tiles")
+    return results
 
 
 def box_muller(words, out=None, stream=None):

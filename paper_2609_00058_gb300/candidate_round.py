@@ -7,17 +7,21 @@ and the reward r = -1 + C + C * V * P (Eq. 4).
 
 A task here is an in-place binary fp32 vector operation, a <- f(a, b), the
 shape of the paper's running example (vecAddInplace).  A candidate is a CUDA
-source exporting
+source defining
 
     extern "C" int candidate_launch(float* a, const float* b, long long n, void* stream);
 
 which enqueues the operation on `stream` and returns 0 (or a CUDA error
 code).  The reference is a source with the same export that the caller
-trusts.  Both are compiled by nvcc into shared libraries (the compilation
-parameters phi of Eq. 2 are the nvcc flags), loaded with ctypes and run on
-device buffers that syn_generate filled; every data-parallel step of the
-round runs on the GPU.  The paper leaves the unit of the latency open: P is
-reported in 1/ms.
+trusts.  Two ways to run them:
+- run_round: both compiled by nvcc into shared libraries (the compilation
+  parameters phi of Eq. 2 are the nvcc flags), loaded with ctypes and run on
+  device buffers that syn_generate filled;
+- run_program_round: both compiled into self-contained programs behind the
+  scaffold's main() (scaffold/vec_inplace_main.h, Sec. 4.1.2), which read
+  their inputs from tensor files named on the command line and write their
+  outputs to files that are loaded back dtype-correctly (sv_read_tensor).
+The paper leaves the unit of the latency open: P is reported in 1/ms.
 """
 from __future__ import annotations
 
@@ -27,11 +31,14 @@ import subprocess
 from dataclasses import dataclass, field
 from typing import List, Optional, Sequence
 
-from . import GenSpec, Pair, decode_results, generate, progressive
+from . import GenSpec, Pair, SynVerifyError, compare, decode_results, generate, progressive, read_tensor, write_tensor
 from .build import ARCH, nvcc
 
 DEFAULT_FLAGS = (*ARCH, "-O3", "-shared", "-Xcompiler", "-fPIC")
+PROGRAM_FLAGS = (*ARCH, "-O3")
 LAUNCH_SYMBOL = "candidate_launch"
+SCAFFOLD_DIR = os.path.join(os.path.dirname(os.path.abspath(__file__)), "scaffold")
+VEC_INPLACE_MAIN = "vec_inplace_main.h"
 
 
 @dataclass
@@ -55,6 +62,7 @@ class Compiled:
     ok: bool  # C of Eq. 2
     path: Optional[str]
     log: str
+    calling_convention: Optional[str] = None  # emitted at compile time (#pragma message)
 
 
 @dataclass
@@ -85,6 +93,30 @@ def compile_kernel(src: str, out_dir: str, flags: Sequence[str] = DEFAULT_FLAGS)
     if p.returncode != 0 or not os.path.exists(out):
         return Compiled(False, None, log)
     return Compiled(True, out, log)
+
+
+def _calling_convention(log: str) -> Optional[str]:
+    for line in log.splitlines():
+        k = line.find("Calling convention:")
+        if k >= 0:
+            return line[k + len("Calling convention:"):].strip().strip("\"'\u2018\u2019")
+    return None
+
+
+def compile_program(src: str, out_dir: str, main_header: str = VEC_INPLACE_MAIN,
+                    flags: Sequence[str] = PROGRAM_FLAGS) -> Compiled:
+    """The compilation tool of Eq. 2 for a self-contained program: the
+    candidate's source compiled behind the scaffold's main() (which reads the
+    test inputs, calls the launcher and writes the outputs, Sec. 4.1.2).  The
+    calling convention the scaffold emits at compile time is returned."""
+    os.makedirs(out_dir, exist_ok=True)
+    out = os.path.join(out_dir, os.path.splitext(os.path.basename(src))[0])
+    p = subprocess.run([nvcc(), *flags, "-I" + SCAFFOLD_DIR, "-include", main_header, "-o", out, src],
+                       capture_output=True, text=True)
+    log = (p.stdout + p.stderr).strip()
+    if p.returncode != 0 or not os.path.exists(out):
+        return Compiled(False, None, log, _calling_convention(log))
+    return Compiled(True, out, log, _calling_convention(log))
 
 
 def _launcher(path: str):
@@ -180,6 +212,76 @@ def run_round(task: Task, candidate_src: str, reference_src: str, work_dir: str,
     return RoundResult(1, 1, p, reward(1, 1, p), latency, -1, stages, cand.log)
 
 
+def run_program_round(task: Task, candidate_src: str, reference_src: str, work_dir: str, runs: int = 20,
+                      timeout: float = 120.0, device=None) -> RoundResult:
+    """One round with self-contained programs exchanging tensor files (the
+    scaffold's process boundary, Sec. 4.1.2): the stage inputs are synthesized
+    on the GPU and written to files; stage by stage, the reference and the
+    candidate program read them, run and write their outputs; the outputs are
+    loaded back dtype-correctly (a file that is not float32 of the stage's
+    size fails the stage) and compared with Eq. 1; the first failing stage
+    ends the round (later stages are not run at all).  P is the candidate
+    program's mean latency over `runs` launches on the largest stage."""
+    import torch
+    cand = compile_program(candidate_src, os.path.join(work_dir, "candidate"))
+    if not cand.ok:
+        return RoundResult(0, 0, 0.0, reward(0, 0, 0.0), None, -1, [], cand.log)
+    ref = compile_program(reference_src, os.path.join(work_dir, "reference"))
+    if not ref.ok:
+        raise RuntimeError("the reference does not compile:\n" + ref.log)
+    dev = torch.device(device or "cuda")
+    layout, nbytes = stage_layout(task)
+    arena = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+    generate(input_specs(task, layout), arena)
+    files = os.path.join(work_dir, "files")
+    os.makedirs(files, exist_ok=True)
+
+    def path(kind, s):
+        return os.path.join(files, "%s_%d.svt" % (kind, s))
+
+    def run(prog, s, out, extra=()):
+        return subprocess.run([prog, path("a", s), path("b", s), out, *extra], capture_output=True, text=True,
+                              timeout=timeout)
+
+    stages: List[dict] = []
+    first_failed = -1
+    for s, (n, (a_off, b_off, r_off, c_off)) in enumerate(zip(task.stages, layout)):
+        write_tensor(path("a", s), arena[a_off: a_off + 4 * n], dtype="f32", shape=(n,))
+        write_tensor(path("b", s), arena[b_off: b_off + 4 * n], dtype="f32", shape=(n,))
+        rr = run(ref.path, s, path("ref", s))
+        if rr.returncode != 0:
+            raise RuntimeError("the reference program failed:\n" + rr.stderr)
+        read_tensor(path("ref", s), file_dtype="f32", n=n, strict=True, out=arena[r_off: r_off + 4 * n])
+        cr = run(cand.path, s, path("cand", s))
+        ok = cr.returncode == 0
+        if ok:
+            try:  # the output must be float32 with the stage's element count
+                read_tensor(path("cand", s), file_dtype="f32", n=n, strict=True, out=arena[c_off: c_off + 4 * n])
+            except SynVerifyError:
+                ok = False
+        if ok:
+            res = decode_results(compare([Pair("f32", n, c_off, r_off, task.atol, task.rtol)], arena, arena), 1)[0]
+        else:
+            res = {"state": 1, "pass": 0, "mismatches": n, "first_mismatch": 0, "max_abs": float("nan"),
+                   "program_error": (cr.stderr or "").strip()[-500:]}
+        stages.append(res)
+        if not res["pass"]:
+            first_failed = s
+            break
+    if first_failed >= 0:
+        return RoundResult(1, 0, 0.0, reward(1, 0, 0.0), None, first_failed, stages, cand.log)
+    last = len(task.stages) - 1
+    cr = run(cand.path, last, path("cand_t", last), (str(runs),))
+    latency = None
+    for line in cr.stdout.splitlines():
+        if line.startswith("latency_ms "):
+            latency = float(line.split()[1])
+    if cr.returncode != 0 or latency is None or latency <= 0:
+        return RoundResult(1, 0, 0.0, reward(1, 0, 0.0), None, last, stages, cand.log)
+    p = 1.0 / latency
+    return RoundResult(1, 1, p, reward(1, 1, p), latency, -1, stages, cand.log)
+
+
 def main(argv=None) -> int:
     """python -m paper_2609_00058_gb300.candidate_round CANDIDATE.cu REFERENCE.cu [--work DIR]:
     one round of the in-place vector task, printed as one JSON line."""
@@ -191,9 +293,12 @@ def main(argv=None) -> int:
     ap.add_argument("reference")
     ap.add_argument("--work", default=None)
     ap.add_argument("--runs", type=int, default=20)
+    ap.add_argument("--programs", action="store_true",
+                    help="run self-contained programs that exchange tensor files instead of shared libraries")
     a = ap.parse_args(argv)
     work = a.work or tempfile.mkdtemp(prefix="candidate_round_")
-    r = run_round(Task("vecAddInplace"), a.candidate, a.reference, work, runs=a.runs)
+    rnd = run_program_round if a.programs else run_round
+    r = rnd(Task("vecAddInplace"), a.candidate, a.reference, work, runs=a.runs)
     print(json.dumps({"C": r.C, "V": r.V, "P_per_ms": r.P, "r": r.r, "latency_ms": r.latency_ms,
                       "first_failed_stage": r.first_failed,
                       "stages": [{k: s[k] for k in ("state", "pass", "mismatches", "first_mismatch", "max_abs")}

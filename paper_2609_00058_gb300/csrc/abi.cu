@@ -18,6 +18,7 @@
 namespace sv {
 
 static_assert(sizeof(sv_perturb) == 40, "sv_perturb layout");
+static_assert(sizeof(vc_tiles) == 88, "vc_tiles layout");
 static_assert(sizeof(syn_spec) == 224, "syn_spec layout");
 static_assert(sizeof(vc_pair) == 48, "vc_pair layout");
 static_assert(sizeof(vc_result) == 80, "vc_result layout");
@@ -172,6 +173,34 @@ static int check_pair(const vc_pair& p, uint64_t cand_bytes, uint64_t ref_bytes)
   int rc;
   if ((rc = check_range(p.cand_offset, bytes, cand_bytes))) return rc;
   if ((rc = check_range(p.ref_offset, bytes, ref_bytes))) return rc;
+  return SV_OK;
+}
+
+// a shaped output: geometry, alignment and both operands inside their buffers
+static int check_tiles(const vc_tiles& t, uint64_t cand_bytes, uint64_t ref_bytes, uint64_t* n_tiles) {
+  if (t.dtype > SV_U32 || (t.flags & ~(uint32_t)SV_EQUAL_NAN)) return SV_EINVAL;
+  if (is_float((int)t.dtype) && !(t.atol >= 0.0 && t.rtol >= 0.0)) return SV_EINVAL;
+  if (t.tile_rows == 0 || t.tile_cols == 0) return SV_EINVAL;
+  if (t.cand_pitch < t.cols || t.ref_pitch < t.cols) return SV_EINVAL;
+  const uint64_t sz = elem_bytes((int)t.dtype);
+  *n_tiles = 0;
+  if (t.rows == 0 || t.cols == 0) return SV_OK;
+  const uint64_t th = t.tile_rows < t.rows ? t.tile_rows : t.rows;
+  const uint64_t tw = t.tile_cols < t.cols ? t.tile_cols : t.cols;
+  if (th > 0x7FFFFFFFull || tw > 0x7FFFFFFFull) return SV_EINVAL;
+  if (t.cand_offset % 16 || t.ref_offset % 16) return SV_EALIGN;
+  if (t.rows > 1 && ((t.cand_pitch * sz) % 16 || (t.ref_pitch * sz) % 16)) return SV_EALIGN;
+  if (t.tile_cols < t.cols && (t.tile_cols * sz) % 16) return SV_EALIGN;
+  // the last element of each operand: offset + ((rows - 1) * pitch + cols) * size, without overflow
+  for (int k = 0; k < 2; ++k) {
+    const uint64_t pitch = k ? t.ref_pitch : t.cand_pitch, off = k ? t.ref_offset : t.cand_offset;
+    const uint64_t buf = k ? ref_bytes : cand_bytes;
+    if (pitch > UINT64_MAX / sz / t.rows) return SV_ERANGE;
+    if (!add_ok(off, ((t.rows - 1) * pitch + t.cols) * sz, buf)) return SV_ERANGE;
+  }
+  const uint64_t ntr = (t.rows + t.tile_rows - 1) / t.tile_rows, ntc = (t.cols + t.tile_cols - 1) / t.tile_cols;
+  if (ntr > SV_MAX_TILES || ntc > SV_MAX_TILES || ntr * ntc > SV_MAX_TILES) return SV_ERANGE;
+  *n_tiles = ntr * ntc;
   return SV_OK;
 }
 
@@ -357,6 +386,29 @@ int syn_box_muller(const uint32_t* d_words, size_t n_pairs, float* d_z, sv_strea
   if (n_pairs > SV_MAX_LOGICAL_N / 2) return SV_ERANGE;
   if ((reinterpret_cast<uintptr_t>(d_words) | reinterpret_cast<uintptr_t>(d_z)) & 7) return SV_EALIGN;
   return status_of(launch_box_muller(d_words, n_pairs, d_z, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int sv_check_tiles(const vc_tiles* tiles, size_t cand_bytes, size_t ref_bytes, uint64_t* n_tiles) {
+  uint64_t n = 0;
+  if (!tiles) return SV_EINVAL;
+  const int rc = check_tiles(*tiles, cand_bytes, ref_bytes, &n);
+  if (n_tiles) *n_tiles = rc == SV_OK ? n : 0;
+  return rc;
+}
+
+int verify_compare_tiles(const vc_tiles* tiles, const void* d_cand, size_t cand_bytes, const void* d_ref,
+                         size_t ref_bytes, vc_result* d_results, sv_stream_t stream) {
+  if (!tiles) return SV_EINVAL;
+  uint64_t n = 0;
+  if (int rc = check_tiles(*tiles, cand_bytes, ref_bytes, &n)) return rc;
+  if (n == 0) return SV_OK;
+  if (!d_cand || !d_ref || !d_results) return SV_EINVAL;
+  if ((reinterpret_cast<uintptr_t>(d_cand) | reinterpret_cast<uintptr_t>(d_ref)) & 15) return SV_EALIGN;
+  if (reinterpret_cast<uintptr_t>(d_results) & 7) return SV_EALIGN;
+  const uint64_t ntc = (tiles->cols + tiles->tile_cols - 1) / tiles->tile_cols;
+  return status_of(launch_compare_tiles(*tiles, ntc, n, static_cast<const uint8_t*>(d_cand),
+                                        static_cast<const uint8_t*>(d_ref), d_results,
+                                        reinterpret_cast<cudaStream_t>(stream)));
 }
 
 const char* sv_strerror(int status) {

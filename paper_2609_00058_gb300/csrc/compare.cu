@@ -543,6 +543,162 @@ __global__ void __launch_bounds__(kThreads) combine_stages_kernel(const __grid_c
 }
 
 // ---------------------------------------------------------------------------
+// shaped outputs: a rows x cols output with row pitches, tile by tile.  One
+// CTA owns a whole tile at a time (grid-stride over the tiles): its threads
+// walk the tile's whole 16-byte vectors in row-major order, U per step, with
+// row / column counters that advance by a constant (no division per vector),
+// then the ragged ends of the rows one element each; the CTA folds the tile
+// and writes its vc_result.  Reported indices are output-wide, row * cols + col.
+// ---------------------------------------------------------------------------
+struct TileParams {
+  vc_tiles t;
+  uint64_t ntc, n_tiles;  // tiles per tile row, tiles in all
+  const uint8_t* cand;
+  const uint8_t* ref;
+  vc_result* results;
+};
+
+// fold b (statistics of other elements) into a; first by minimum
+__device__ __forceinline__ void acc_merge(Acc& a, const Acc& b) {
+  a.mism += b.mism;
+  a.nan_d += b.nan_d;
+  a.inf_d += b.inf_d;
+  a.nonfin += b.nonfin;
+  a.first = b.first < a.first ? b.first : a.first;
+  a.ssq += b.ssq;
+  a.maxabs_f = fmaxf(a.maxabs_f, b.maxabs_f);
+  a.maxrel_f = fmaxf(a.maxrel_f, b.maxrel_f);
+  a.relthr = fmaxf(a.relthr, b.relthr);
+  a.maxabs_u = b.maxabs_u > a.maxabs_u ? b.maxabs_u : a.maxabs_u;
+  a.maxrel_d = fmax(a.maxrel_d, b.maxrel_d);
+}
+
+__device__ __forceinline__ vc_result tile_result(const Partial& q, uint64_t n, bool fl) {
+  vc_result r;
+  r.mismatches = q.mism;
+  r.nan_disagree = q.nan_d;
+  r.inf_disagree = q.inf_d;
+  r.n_finite = fl ? n - q.nonfin : n;
+  r.first_mismatch = q.first == ~0ull ? -1 : (int64_t)q.first;
+  r.max_abs_u64 = fl ? 0 : q.maxabs;
+  r.max_abs = fl ? (double)__uint_as_float((uint32_t)q.maxabs) : (double)q.maxabs;
+  r.max_rel = q.maxrel;
+  r.rms = r.n_finite ? sqrt(q.ssq / (double)r.n_finite) : 0.0;
+  r.pass = q.mism == 0;
+  r.state = SV_STAGE_RUN;
+  return r;
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant__ TileParams p) {
+  constexpr uint32_t sz = elem_bytes(DT), VE = 16 / sz;
+  constexpr int U = kCmpTileBytes / 16 / kThreads;  // vectors per thread per step (4)
+  constexpr uint32_t kStep = (uint32_t)U * kThreads;
+  __shared__ Partial tile_sum;
+  const vc_tiles& t = p.t;
+  const Tol tol{__double2float_rn(t.atol), __double2float_rn(t.rtol), (t.flags & SV_EQUAL_NAN) != 0};
+  const uint8_t* xb = p.cand + t.cand_offset;
+  const uint8_t* yb = p.ref + t.ref_offset;
+  for (uint64_t tile = blockIdx.x; tile < p.n_tiles; tile += gridDim.x) {
+    const uint64_t ti = tile / p.ntc, tj = tile - ti * p.ntc;
+    const uint64_t r0 = ti * t.tile_rows, c0 = tj * t.tile_cols;
+    const uint32_t h = (uint32_t)(umin(r0 + t.tile_rows, t.rows) - r0);
+    const uint32_t w = (uint32_t)(umin(c0 + t.tile_cols, t.cols) - c0);
+    const uint32_t vr = w / VE;  // whole vectors per row of the tile
+    Acc a;
+    acc_reset(a);
+    if (vr > 0) {
+      uint32_t rr[U], cc[U];  // row and vector column (in the tile) of this thread's u-th vector
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const uint32_t v = threadIdx.x + (uint32_t)u * kThreads;
+        rr[u] = v / vr;
+        cc[u] = v - rr[u] * vr;
+      }
+      const uint32_t dq = kStep / vr, dr = kStep - dq * vr;
+      const uint64_t nvec = (uint64_t)h * vr;
+      for (uint64_t base = 0; base < nvec; base += kStep) {  // uniform trip count: the shuffles below need the warp
+        uint4 x[U], y[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          if (rr[u] < h) {
+            const uint64_t row = r0 + rr[u], col = c0 + (uint64_t)cc[u] * VE;
+            x[u] = ldg_stream(reinterpret_cast<const uint4*>(xb + (row * t.cand_pitch + col) * sz));
+            y[u] = ldg_stream(reinterpret_cast<const uint4*>(yb + (row * t.ref_pitch + col) * sz));
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          if (rr[u] < h) do_vector<DT>(a, tol, x[u], y[u], (r0 + rr[u]) * t.cols + c0 + (uint64_t)cc[u] * VE);
+          cc[u] += dr;
+          rr[u] += dq;
+          if (cc[u] >= vr) {
+            cc[u] -= vr;
+            ++rr[u];
+          }
+        }
+        if constexpr (is_float(DT)) {  // share the running max |x-y|/|y| across the warp (as cmp_run)
+          float m = a.maxrel_f;
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+          a.relthr = __fmul_rn(m, 1.0f - 0x1p-20f);
+        }
+      }
+    }
+    if (vr * VE < w) {  // the ragged end of every row: one thread per row, elements in order
+      Acc b;
+      acc_reset(b);
+      for (uint32_t r = threadIdx.x; r < h; r += kThreads) {
+        const uint64_t row = r0 + r, cs = c0 + (uint64_t)vr * VE;
+        Acc e;
+        acc_reset(e);
+        do_tail<DT>(e, tol, xb + (row * t.cand_pitch + cs) * sz, yb + (row * t.ref_pitch + cs) * sz, 0,
+                    w - vr * VE);
+        if (e.first != ~0ull) e.first += row * t.cols + cs;  // do_tail reports indices from 0
+        acc_merge(b, e);
+      }
+      acc_merge(a, b);
+    }
+    flush<is_float(DT)>(a, &tile_sum);  // block fold; ends with a barrier
+    if (threadIdx.x == 0) p.results[tile] = tile_result(tile_sum, (uint64_t)h * w, is_float(DT));
+  }
+}
+
+static const void* tile_kernel_for(uint32_t dtype) {
+  switch (dtype) {
+    case SV_F32: return reinterpret_cast<const void*>(&tile_kernel<SV_F32>);
+    case SV_F16: return reinterpret_cast<const void*>(&tile_kernel<SV_F16>);
+    case SV_BF16: return reinterpret_cast<const void*>(&tile_kernel<SV_BF16>);
+    case SV_I32: return reinterpret_cast<const void*>(&tile_kernel<SV_I32>);
+    case SV_I64: return reinterpret_cast<const void*>(&tile_kernel<SV_I64>);
+    default: return reinterpret_cast<const void*>(&tile_kernel<SV_U32>);
+  }
+}
+
+cudaError_t launch_compare_tiles(const vc_tiles& t, uint64_t ntc, uint64_t n_tiles, const uint8_t* cand,
+                                 const uint8_t* ref, vc_result* results, cudaStream_t st) {
+  if (n_tiles == 0) return cudaSuccess;
+  TileParams tp;
+  tp.t = t;
+  tp.ntc = ntc;
+  tp.n_tiles = n_tiles;
+  tp.cand = cand;
+  tp.ref = ref;
+  tp.results = results;
+  const uint32_t grid = (uint32_t)umin(n_tiles, grid_cap_for(tile_kernel_for(t.dtype)));
+  switch (t.dtype) {
+    case SV_F32: tile_kernel<SV_F32><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_F16: tile_kernel<SV_F16><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_BF16: tile_kernel<SV_BF16><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_I32: tile_kernel<SV_I32><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_I64: tile_kernel<SV_I64><<<grid, launch_block(), 0, st>>>(tp); break;
+    default: tile_kernel<SV_U32><<<grid, launch_block(), 0, st>>>(tp); break;
+  }
+  count_launch();
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // host launchers
 // ---------------------------------------------------------------------------
 static const void* cmp_kernel_for(uint32_t dtype) {

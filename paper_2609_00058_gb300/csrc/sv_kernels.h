@@ -140,6 +140,10 @@ cudaError_t launch_compare_small(const DevPair* host, const DevPair* dev, int n,
 cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const Partial* partials,
                            vc_result* results, int32_t* flag, int first_group, cudaStream_t st);
 
+// shaped outputs: one CTA per tile (grid-stride); ntc tiles per tile row
+cudaError_t launch_compare_tiles(const vc_tiles& t, uint64_t ntc, uint64_t n_tiles, const uint8_t* cand,
+                                 const uint8_t* ref, vc_result* results, cudaStream_t st);
+
 // ---- value conversion of test data (convert.cu) ----
 // n elements of type s at src become n elements of type d at dst (16-byte
 // aligned, s != d, not float -> integer); clamped or overflowed values are

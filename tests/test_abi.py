@@ -202,3 +202,40 @@ def test_failure_hook_arguments():
     lib = sv.lib()
     assert lib.sv_debug_fail_launches(-1) == -1
     assert lib.sv_debug_fail_launches(0) == 0
+
+
+def _tiles(**kw):
+    base = dict(dtype="f32", rows=10, cols=16, cand_offset=0, ref_offset=0, tile_rows=4, tile_cols=8)
+    base.update(kw)
+    return W.Tiles(**base)
+
+
+BAD_TILES = [
+    (dict(dtype="f32", atol=-1.0), -1),
+    (dict(tile_rows=0), -1),
+    (dict(cand_pitch=15), -1),                         # pitch below cols
+    (dict(cand_offset=8), -2),
+    (dict(cand_pitch=17), -2),                         # pitch * 4 bytes not a multiple of 16
+    (dict(tile_cols=6), -2),                           # tile width not whole vectors
+    (dict(rows=10, ref_pitch=1 << 20), -3),            # the reference beyond its buffer
+    (dict(rows=1 << 20, cols=1 << 16, tile_rows=1, tile_cols=4), -3),  # beyond the buffers, and 2^34 tiles
+]
+
+
+@pytest.mark.parametrize("kw,rc", BAD_TILES)
+def test_tile_validation(lib, kw, rc):
+    t = _tiles(**kw)
+    n = C.c_uint64(7)
+    got = lib.sv_check_tiles(C.byref(sv.to_c_tiles(t)), 1 << 20 if rc != -3 else 4096, 4096 * 16, C.byref(n))
+    assert got == rc and n.value == 0
+
+
+def test_tile_counts(lib):
+    assert sv.tile_count(_tiles()) == 3 * 2
+    assert sv.tile_count(_tiles(rows=0)) == 0
+    assert sv.tile_count(_tiles(tile_rows=1, tile_cols=16)) == 10
+    assert sv.tile_count(_tiles(rows=1, cols=3, tile_cols=3)) == 1  # one row, narrower than a vector: no pitch rule
+    assert sv.tile_count(_tiles(rows=1 << 16, cols=1 << 16, tile_rows=1, tile_cols=4, cand_pitch=0, ref_pitch=0),
+                         1 << 34, 1 << 34) == 1 << 30
+    with pytest.raises(sv.SynVerifyError):
+        sv.tile_count(_tiles(tile_cols=6))

@@ -95,3 +95,38 @@ def test_fault_found_at_the_right_stage_on_other_ladders(tmp_path):
     assert r.first_failed == 2
     assert [s["state"] for s in r.stages] == [sv.STAGE_RUN] * 3 + [sv.STAGE_SKIPPED]
     assert r.stages[2]["mismatches"] <= 1 and r.stages[2]["first_mismatch"] in (-1, 1 << 20)
+
+
+# ---------------------------------------------------------------------------
+# self-contained programs exchanging tensor files (the scaffold's process boundary)
+# ---------------------------------------------------------------------------
+def test_broken_program_scores_minus_one(tmp_path):
+    r = cr.run_program_round(TASK, src("vec_add_inplace_broken"), src("vec_add_reference"), str(tmp_path))
+    assert (r.C, r.V, r.r) == (0, 0, -1.0)
+
+
+@pytest.mark.gpu
+def test_correct_program_round(tmp_path):
+    from gpu_util import device
+    device()
+    r = cr.run_program_round(TASK, src("vec_add_inplace"), src("vec_add_reference"), str(tmp_path))
+    assert (r.C, r.V, r.first_failed) == (1, 1, -1)
+    assert r.latency_ms > 0 and r.r == r.P == pytest.approx(1.0 / r.latency_ms)
+    assert len(r.stages) == len(TASK.stages) and all(s["pass"] and s["mismatches"] == 0 for s in r.stages)
+    # the files the programs exchanged are tensor files of the stage sizes
+    import tensor_files as TF
+    name, shape, data = TF.parse(os.path.join(str(tmp_path), "files", "cand_3.svt"))
+    assert (name, shape) == ("f32", (TASK.stages[3],))
+
+
+@pytest.mark.gpu
+def test_faulty_program_stops_at_the_failing_stage(tmp_path):
+    """Fail-fast across processes: stage 3 fails, and no later stage is run."""
+    from gpu_util import device
+    device()
+    task = cr.Task("vecAddInplace", stages=(1000, 1 << 16, 1 << 21, 1 << 22), seed=3)
+    r = cr.run_program_round(task, src("vec_add_inplace_faulty"), src("vec_add_reference"), str(tmp_path))
+    assert (r.C, r.V, r.r, r.first_failed) == (1, 0, 0.0, 2)
+    assert [s["pass"] for s in r.stages] == [True, True, False]
+    assert r.stages[2]["first_mismatch"] >= 1 << 20
+    assert not os.path.exists(os.path.join(str(tmp_path), "files", "a_3.svt"))

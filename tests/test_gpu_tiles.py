@@ -1,0 +1,133 @@
+"""Parity of verify_compare_tiles (shaped outputs compared tile by tile) with
+the oracle's or_compare_tiles, through the C ABI on the GPU: every dtype,
+dense and padded pitches (different per operand), tiles that divide the
+output and ragged ones, tiles narrower than a 16-byte vector, one row per
+tile, one tile for everything; planted mismatches, NaN, infinities and
+denormals; and the dot-like workload's 32768 x 32768 bf16 output in
+128 x 128 tiles, checked on sampled tile rows the oracle computes."""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2609_00058_gb300 as sv
+import workloads as W
+from gpu_util import assert_results_match, device, to_dev
+
+pytestmark = pytest.mark.gpu
+NP = {"f32": np.float32, "f16": np.float16, "i32": np.int32, "i64": np.int64, "u32": np.uint32}
+
+
+@pytest.fixture(scope="module")
+def dev():
+    return device()
+
+
+def make_pair(dtype, rows, cols, cpitch, rpitch, seed):
+    """Reference and candidate of a rows x cols output in buffers with the given
+    pitches; padding holds garbage that differs between the two."""
+    rng = np.random.default_rng(seed)
+    if dtype == "bf16":
+        vals = rng.normal(5, 10, size=(rows, cols)).astype(np.float32)
+        yv = (vals.view(np.uint32) >> 16).astype(np.uint16)
+        xv = yv.copy()
+        flat = xv.reshape(-1)
+        k = rng.choice(flat.size, max(1, flat.size // 500), replace=False)
+        flat[k] ^= rng.integers(1, 1 << 8, size=k.size, dtype=np.uint16)
+        flat[rng.choice(flat.size, 3)] = 0x7FC0
+        store = np.uint16
+    elif dtype in ("f32", "f16"):
+        yv = rng.normal(5, 10, size=(rows, cols)).astype(NP[dtype])
+        xv = (yv + rng.normal(0, 1e-3, size=yv.shape).astype(NP[dtype])).astype(NP[dtype])
+        flat, yflat = xv.reshape(-1), yv.reshape(-1)
+        flat[rng.choice(flat.size, max(1, flat.size // 300), replace=False)] += 1
+        flat[rng.choice(flat.size, 2)] = np.nan
+        yflat[rng.choice(flat.size, 2)] = np.inf
+        flat[rng.choice(flat.size, 2)] = np.finfo(NP[dtype]).tiny / 4
+        store = NP[dtype]
+    else:
+        info = np.iinfo(NP[dtype])
+        yv = rng.integers(max(info.min, -1000), min(info.max, 1000), size=(rows, cols), dtype=NP[dtype])
+        xv = yv.copy()
+        flat = xv.reshape(-1)
+        flat[rng.choice(flat.size, max(1, flat.size // 400), replace=False)] = info.max
+        store = NP[dtype]
+    x = np.full((rows, cpitch), 0x55, dtype=np.uint8 if store is None else store)
+    y = np.full((rows, rpitch), 0x33, dtype=x.dtype)
+    x[:, :cols] = xv.view(x.dtype)
+    y[:, :cols] = yv.view(y.dtype)
+    return np.ascontiguousarray(x).view(np.uint8).reshape(-1), np.ascontiguousarray(y).view(np.uint8).reshape(-1)
+
+
+CASES = [  # rows, cols, cand pitch, ref pitch, tile rows, tile cols
+    (64, 256, 256, 256, 16, 64),
+    (37, 100, 104, 112, 8, 32),      # ragged in both directions, padded pitches
+    (5, 1000, 1000, 1024, 1, 1000),  # one row per tile
+    (33, 36, 36, 40, 33, 36),        # one tile
+    (50, 24, 24, 24, 7, 8),          # tiles of two 16-byte vectors
+    (9, 3, 4, 8, 2, 3),              # rows narrower than a vector: ragged ends only
+    (300, 513, 520, 520, 128, 128),
+]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f16", "bf16", "i32", "i64", "u32"])
+@pytest.mark.parametrize("case", CASES)
+def test_tiles_match_oracle(dev, dtype, case):
+    rows, cols, cp, rp, tr, tc = case
+    sz = W.DTYPE_BYTES[dtype]
+    align = 16 // sz  # pitches and tile widths in whole 16-byte vectors (the ABI's alignment rule)
+    cp, rp = -(-cp // align) * align, -(-rp // align) * align
+    if tc < cols:
+        tc = -(-tc // align) * align
+    x, y = make_pair(dtype, rows, cols, cp, rp, seed=rows * 7 + cols)
+    t = W.Tiles(dtype, rows, cols, 0, 0, cand_pitch=cp, ref_pitch=rp, tile_rows=tr, tile_cols=tc,
+                atol=1e-3, rtol=1e-3)
+    want = oracle.compare_tiles(t, x, y)
+    res = sv.compare_tiles(t, to_dev(x, dev), to_dev(y, dev))
+    got = sv.decode_results(res, len(want))
+    assert_results_match(got, want, "%s %r" % (dtype, case))
+    assert any(not w["pass"] for w in want)
+
+
+def test_offsets_and_shared_buffer(dev):
+    """Both operands in one arena at 16-byte aligned offsets, a sub-matrix view."""
+    rows, cols = 40, 64
+    x, y = make_pair("f32", rows, 96, 96, 96, seed=5)
+    arena = np.zeros(4096 + x.size + y.size + 64, np.uint8)
+    arena[4096:4096 + x.size], arena[4096 + x.size + 48: 4096 + x.size + 48 + y.size] = x, y
+    t = W.Tiles("f32", rows, cols, 4096 + 16 * 4, 4096 + x.size + 48 + 16 * 4, cand_pitch=96, ref_pitch=96,
+                tile_rows=16, tile_cols=16, atol=1e-4, rtol=1e-4)  # columns 16..79 of each operand
+    want = oracle.compare_tiles(t, arena, arena)
+    a = to_dev(arena, dev)
+    assert_results_match(sv.decode_results(sv.compare_tiles(t, a, a), len(want)), want, "sub-matrix")
+
+
+def test_dotlike_output_per_tile(dev):
+    """The dot-like workload's bf16 32768 x 32768 reference and its noisy twin,
+    compared in 128 x 128 tiles (65536 results); sampled tile rows are
+    recomputed by the oracle from the same bytes."""
+    import torch
+    wl = W.FULL_SIZE["dotlike_bf16"]()
+    arena = torch.zeros(wl.arena_bytes, dtype=torch.uint8, device=dev)
+    for call in wl.gen_calls:
+        sv.generate(call, arena)
+    pr = wl.pairs[0]
+    side = 1 << 15
+    t = W.Tiles("bf16", side, side, pr.cand_offset, pr.ref_offset, tile_rows=128, tile_cols=128,
+                atol=pr.atol, rtol=pr.rtol)
+    res = sv.compare_tiles(t, arena, arena)
+    got = sv.decode_results(res, 256 * 256)
+    whole = sv.decode_results(sv.compare([pr], arena, arena), 1)[0]
+    assert sum(g["mismatches"] for g in got) == whole["mismatches"]
+    assert sum(g["n_finite"] for g in got) == whole["n_finite"] == side * side
+    firsts = [g["first_mismatch"] for g in got if g["first_mismatch"] >= 0]
+    assert (min(firsts) if firsts else -1) == whole["first_mismatch"]
+    for ti in (0, 97, 255):  # one tile row each: rows [128 ti, 128 ti + 128)
+        rows0 = 128 * ti * side * 2
+        c = arena[pr.cand_offset + rows0: pr.cand_offset + rows0 + 128 * side * 2].cpu().numpy()
+        r = arena[pr.ref_offset + rows0: pr.ref_offset + rows0 + 128 * side * 2].cpu().numpy()
+        sub = W.Tiles("bf16", 128, side, 0, 0, tile_rows=128, tile_cols=128, atol=pr.atol, rtol=pr.rtol)
+        want = oracle.compare_tiles(sub, c, r)
+        for w in want:  # the oracle's indices are relative to the sampled rows
+            if w["first_mismatch"] >= 0:
+                w["first_mismatch"] += 128 * ti * side
+        assert_results_match(got[256 * ti: 256 * ti + 256], want, "tile row %d" % ti)
