@@ -411,6 +411,30 @@ def ours_arm(args, rank, world):
         cand_pass = {"what": "candidate pass alone: reference read, noisy twin written", "ms": cp_ms,
                      "bytes": cp_bytes, "gbs": cp_bytes / (cp_ms * 1e-3) / 1e9}
 
+    # the dot-like output compared per 128 x 128 tile (shaped outputs): the
+    # same bytes as the verify step, 65536 verdicts instead of one
+    tile_pass = None
+    if args.workload == "dotlike_bf16":
+        pr = wl.pairs[0]
+        side = int(round(pr.n ** 0.5))
+        tt = sv.Tiles(pr.dtype, side, side, pr.cand_offset, pr.ref_offset, tile_rows=128, tile_cols=128,
+                      atol=pr.atol, rtol=pr.rtol)
+        n_t = sv.tile_count(tt, wl.arena_bytes, wl.arena_bytes)
+        tres = torch.empty(n_t * sv.RESULT_BYTES, dtype=torch.uint8, device=dev)
+        for _ in range(3):
+            sv.compare_tiles(tt, arena, arena, results=tres)
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        c0.record(stream)
+        for _ in range(args.steps):
+            sv.compare_tiles(tt, arena, arena, results=tres)
+        c1.record(stream)
+        torch.cuda.synchronize()
+        tp_ms = c0.elapsed_time(c1) / args.steps
+        tp_bytes = 2 * pr.n * W.DTYPE_BYTES[pr.dtype]
+        tile_pass = {"what": "verify_compare_tiles, %d x %d output in 128 x 128 tiles (%d verdicts)" % (side, side, n_t),
+                     "ms": tp_ms, "bytes": tp_bytes, "gbs": tp_bytes / (tp_ms * 1e-3) / 1e9}
+
     # end to end: synthesized data delivered to pinned host buffers, verdicts read back
     host = torch.empty(wl.arena_bytes, dtype=torch.uint8, pin_memory=True)
     host_res = torch.empty(results.numel(), dtype=torch.uint8, pin_memory=True)
@@ -513,6 +537,7 @@ def ours_arm(args, rank, world):
         "step_ms_best": min(step_each),
         "roofline": roofline,
         **({"candidate_pass": dict(cand_pass, frac_of_hbm=cand_pass["gbs"] / hbm)} if cand_pass else {}),
+        **({"tile_verify": dict(tile_pass, frac_of_hbm=tile_pass["gbs"] / hbm)} if tile_pass else {}),
         "e2e": {"value": job_throughput(step_bytes, e2e_steps, world, e2e_s), "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps},
         "clocks": clocks,

@@ -95,6 +95,29 @@ class Pair:
     equal_nan: bool = True
 
 
+@dataclass
+class Tiles:
+    """A shaped output (rows x cols, row-major) compared tile by tile; zero
+    pitches and a zero tile_cols mean cols."""
+    dtype: str
+    rows: int
+    cols: int
+    cand_offset: int
+    ref_offset: int
+    cand_pitch: int = 0
+    ref_pitch: int = 0
+    tile_rows: int = 1
+    tile_cols: int = 0
+    atol: float = 0.0
+    rtol: float = 0.0
+    equal_nan: bool = True
+
+    def __post_init__(self):
+        self.cand_pitch = self.cand_pitch or self.cols
+        self.ref_pitch = self.ref_pitch or self.cols
+        self.tile_cols = self.tile_cols or self.cols
+
+
 # ---------------------------------------------------------------------------
 # C structs (layouts of synverify.h)
 # ---------------------------------------------------------------------------

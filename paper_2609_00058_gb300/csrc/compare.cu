@@ -57,7 +57,7 @@ struct Acc {
   uint64_t first;
   double ssq;
   float maxabs_f, maxrel_f;  // float types
-  float relthr;              // float types: maxrel_f * (1 - 2^-20), see float_elem
+  float relthr;              // float types: a max |x-y|/|y| already reached (the warp's), see float_vector
   uint64_t maxabs_u;         // integer types
   double maxrel_d;           // integer types
 };
@@ -89,8 +89,10 @@ struct Tol {
 // registers on the hot path.
 //
 // max |x-y|/|y| stays exact without a division per element: fl(d/|y|) is
-// monotone in the exact quotient, so an element can raise the running maximum
-// M only if d/|y| > M, which implies d > fl(M (1 - 2^-20) |y|).
+// monotone in the exact quotient, so an element can raise a maximum M already
+// reached only if d/|y| > M, that is d - M |y| > 0, and one fused
+// multiply-add gives the sign of d - M |y| exactly (one rounding of the exact
+// value); only those elements are divided.
 //
 // The sum of squares (a statistic, not part of the verdict) accumulates with a
 // fused multiply-add per element, then per 16-byte vector into fp64.
@@ -137,9 +139,9 @@ __device__ __forceinline__ void float_elem_full(Acc& a, const Tol& t, float x, f
     a.ssq = (double)d;
     a.maxrel_f = d;
     a.relthr = d;
-  } else if (ay != 0.0f && d > __fmul_rn(a.relthr, ay)) {
+  } else if (ay != 0.0f && __fmaf_rn(-a.relthr, ay, d) > 0.0f) {
     a.maxrel_f = fmaxf(a.maxrel_f, __fdiv_rn(d, ay));
-    a.relthr = __fmul_rn(a.maxrel_f, 1.0f - 0x1p-20f);
+    a.relthr = a.maxrel_f;
   }
 }
 
@@ -182,7 +184,7 @@ __device__ __forceinline__ void float_vector(Acc& a, const Tol& t, const uint4& 
     const float d = fabsf(__fsub_rn(x[j], y[j]));
     const float tol = __fadd_rn(t.atol, __fmul_rn(t.rtol, ay));
     const bool fin = d <= FLT_MAX;
-    rare |= !(d <= tol) | !fin | (d > __fmul_rn(a.relthr, ay));
+    rare |= !(d <= tol) | !fin | (__fmaf_rn(-a.relthr, ay, d) > 0.0f);
     dk[j] = fin ? d : 0.0f;
     vmax = fmaxf(vmax, dk[j]);
     vsum = __fmaf_rn(dk[j], dk[j], vsum);
@@ -320,7 +322,7 @@ __device__ void cmp_run(Acc& a, const vc_pair& pr, const uint8_t* cand, const ui
       float m = a.maxrel_f;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
-      a.relthr = __fmul_rn(m, 1.0f - 0x1p-20f);
+      a.relthr = m;
     }
   }
   const uint64_t tail0 = vfull * VE;
@@ -589,21 +591,32 @@ __device__ __forceinline__ vc_result tile_result(const Partial& q, uint64_t n, b
   return r;
 }
 
-template <int DT>
+// A team of NT threads owns one tile at a time: the whole CTA (NT = 256) when
+// tiles are few and large, or one warp (NT = 32) when there are many, so that
+// the warps of an SM stream their tiles independently (a warp's fold needs no
+// block barrier, and no tile boundary drains the memory pipeline).
+template <int DT, int NT>
 __global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant__ TileParams p) {
   constexpr uint32_t sz = elem_bytes(DT), VE = 16 / sz;
-  constexpr int U = kCmpTileBytes / 16 / kThreads;  // vectors per thread per step (4)
-  constexpr uint32_t kStep = (uint32_t)U * kThreads;
+  constexpr int U = 4;                                // vectors per thread per step
+  constexpr uint32_t kStep = (uint32_t)U * NT;
+  constexpr int kTeams = kThreads / NT;               // teams per CTA
   __shared__ Partial tile_sum;
+  const int tid = (int)(threadIdx.x % NT);
+  const uint64_t team = (uint64_t)blockIdx.x * kTeams + threadIdx.x / NT;
+  const uint64_t teams = (uint64_t)gridDim.x * kTeams;
   const vc_tiles& t = p.t;
   const Tol tol{__double2float_rn(t.atol), __double2float_rn(t.rtol), (t.flags & SV_EQUAL_NAN) != 0};
   const uint8_t* xb = p.cand + t.cand_offset;
   const uint8_t* yb = p.ref + t.ref_offset;
-  for (uint64_t tile = blockIdx.x; tile < p.n_tiles; tile += gridDim.x) {
-    const uint64_t ti = tile / p.ntc, tj = tile - ti * p.ntc;
+  // every team runs the same number of rounds (a CTA's barrier needs all its threads)
+  const uint64_t rounds = NT == kThreads ? (p.n_tiles + teams - 1) / teams : 0;
+  for (uint64_t k = 0, tile = team; NT == kThreads ? k < rounds : tile < p.n_tiles; ++k, tile += teams) {
+    const bool live = tile < p.n_tiles;
+    const uint64_t ti = live ? tile / p.ntc : 0, tj = live ? tile - ti * p.ntc : 0;
     const uint64_t r0 = ti * t.tile_rows, c0 = tj * t.tile_cols;
-    const uint32_t h = (uint32_t)(umin(r0 + t.tile_rows, t.rows) - r0);
-    const uint32_t w = (uint32_t)(umin(c0 + t.tile_cols, t.cols) - c0);
+    const uint32_t h = live ? (uint32_t)(umin(r0 + t.tile_rows, t.rows) - r0) : 0;
+    const uint32_t w = live ? (uint32_t)(umin(c0 + t.tile_cols, t.cols) - c0) : 0;
     const uint32_t vr = w / VE;  // whole vectors per row of the tile
     Acc a;
     acc_reset(a);
@@ -611,7 +624,7 @@ __global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant
       uint32_t rr[U], cc[U];  // row and vector column (in the tile) of this thread's u-th vector
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const uint32_t v = threadIdx.x + (uint32_t)u * kThreads;
+        const uint32_t v = (uint32_t)tid + (uint32_t)u * NT;
         rr[u] = v / vr;
         cc[u] = v - rr[u] * vr;
       }
@@ -641,14 +654,14 @@ __global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant
           float m = a.maxrel_f;
 #pragma unroll
           for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
-          a.relthr = __fmul_rn(m, 1.0f - 0x1p-20f);
+          a.relthr = m;
         }
       }
     }
     if (vr * VE < w) {  // the ragged end of every row: one thread per row, elements in order
       Acc b;
       acc_reset(b);
-      for (uint32_t r = threadIdx.x; r < h; r += kThreads) {
+      for (uint32_t r = (uint32_t)tid; r < h; r += NT) {
         const uint64_t row = r0 + r, cs = c0 + (uint64_t)vr * VE;
         Acc e;
         acc_reset(e);
@@ -659,19 +672,37 @@ __global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant
       }
       acc_merge(a, b);
     }
-    flush<is_float(DT)>(a, &tile_sum);  // block fold; ends with a barrier
-    if (threadIdx.x == 0) p.results[tile] = tile_result(tile_sum, (uint64_t)h * w, is_float(DT));
+    if constexpr (NT == kThreads) {
+      flush<is_float(DT)>(a, &tile_sum);  // block fold; ends with a barrier
+      if (threadIdx.x == 0 && live) p.results[tile] = tile_result(tile_sum, (uint64_t)h * w, is_float(DT));
+    } else {
+      const Partial f = warp_fold<is_float(DT)>(a);
+      if (tid == 0) p.results[tile] = tile_result(f, (uint64_t)h * w, is_float(DT));
+    }
   }
 }
 
+template <int NT>
 static const void* tile_kernel_for(uint32_t dtype) {
   switch (dtype) {
-    case SV_F32: return reinterpret_cast<const void*>(&tile_kernel<SV_F32>);
-    case SV_F16: return reinterpret_cast<const void*>(&tile_kernel<SV_F16>);
-    case SV_BF16: return reinterpret_cast<const void*>(&tile_kernel<SV_BF16>);
-    case SV_I32: return reinterpret_cast<const void*>(&tile_kernel<SV_I32>);
-    case SV_I64: return reinterpret_cast<const void*>(&tile_kernel<SV_I64>);
-    default: return reinterpret_cast<const void*>(&tile_kernel<SV_U32>);
+    case SV_F32: return reinterpret_cast<const void*>(&tile_kernel<SV_F32, NT>);
+    case SV_F16: return reinterpret_cast<const void*>(&tile_kernel<SV_F16, NT>);
+    case SV_BF16: return reinterpret_cast<const void*>(&tile_kernel<SV_BF16, NT>);
+    case SV_I32: return reinterpret_cast<const void*>(&tile_kernel<SV_I32, NT>);
+    case SV_I64: return reinterpret_cast<const void*>(&tile_kernel<SV_I64, NT>);
+    default: return reinterpret_cast<const void*>(&tile_kernel<SV_U32, NT>);
+  }
+}
+
+template <int NT>
+static void launch_tiles(const TileParams& tp, uint32_t grid, cudaStream_t st) {
+  switch (tp.t.dtype) {
+    case SV_F32: tile_kernel<SV_F32, NT><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_F16: tile_kernel<SV_F16, NT><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_BF16: tile_kernel<SV_BF16, NT><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_I32: tile_kernel<SV_I32, NT><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_I64: tile_kernel<SV_I64, NT><<<grid, launch_block(), 0, st>>>(tp); break;
+    default: tile_kernel<SV_U32, NT><<<grid, launch_block(), 0, st>>>(tp); break;
   }
 }
 
@@ -685,14 +716,15 @@ cudaError_t launch_compare_tiles(const vc_tiles& t, uint64_t ntc, uint64_t n_til
   tp.cand = cand;
   tp.ref = ref;
   tp.results = results;
-  const uint32_t grid = (uint32_t)umin(n_tiles, grid_cap_for(tile_kernel_for(t.dtype)));
-  switch (t.dtype) {
-    case SV_F32: tile_kernel<SV_F32><<<grid, launch_block(), 0, st>>>(tp); break;
-    case SV_F16: tile_kernel<SV_F16><<<grid, launch_block(), 0, st>>>(tp); break;
-    case SV_BF16: tile_kernel<SV_BF16><<<grid, launch_block(), 0, st>>>(tp); break;
-    case SV_I32: tile_kernel<SV_I32><<<grid, launch_block(), 0, st>>>(tp); break;
-    case SV_I64: tile_kernel<SV_I64><<<grid, launch_block(), 0, st>>>(tp); break;
-    default: tile_kernel<SV_U32><<<grid, launch_block(), 0, st>>>(tp); break;
+  // one warp per tile once there are enough tiles for every resident warp to
+  // hold a few; otherwise the whole CTA shares each tile
+  const uint32_t cap_w = grid_cap_for(tile_kernel_for<32>(t.dtype));
+  const bool warps = n_tiles >= 4ull * cap_w * (kThreads / 32);
+  if (warps) {
+    const uint64_t want = (n_tiles + kThreads / 32 - 1) / (kThreads / 32);
+    launch_tiles<32>(tp, (uint32_t)umin(want, cap_w), st);
+  } else {
+    launch_tiles<kThreads>(tp, (uint32_t)umin(n_tiles, grid_cap_for(tile_kernel_for<kThreads>(t.dtype))), st);
   }
   count_launch();
   return cudaGetLastError();

@@ -66,6 +66,8 @@ CASES = [  # rows, cols, cand pitch, ref pitch, tile rows, tile cols
     (50, 24, 24, 24, 7, 8),          # tiles of two 16-byte vectors
     (9, 3, 4, 8, 2, 3),              # rows narrower than a vector: ragged ends only
     (300, 513, 520, 520, 128, 128),
+    (10000, 64, 64, 72, 1, 64),      # enough tiles for one warp per tile
+    (12000, 37, 40, 48, 1, 37),      # one warp per tile, a ragged end in every row
 ]
 
 
@@ -131,3 +133,38 @@ def test_dotlike_output_per_tile(dev):
             if w["first_mismatch"] >= 0:
                 w["first_mismatch"] += 128 * ti * side
         assert_results_match(got[256 * ti: 256 * ti + 256], want, "tile row %d" % ti)
+
+
+def test_manifest_plan_end_to_end(dev):
+    """A manifest entry's plan on the GPU: inputs synthesized with the
+    broad-range preset, a reference output (a copy of input a, as an identity
+    kernel would write it) and a candidate with two planted errors, compared
+    per 32 x 64 tile; the failing tiles are the ones holding the errors, and
+    every tile's verdict equals the oracle's on the same bytes."""
+    import json
+
+    import torch
+
+    from paper_2609_00058_gb300 import manifest as M
+    entry = M.load(json.dumps({
+        "kernel": "identity", "atol": 1e-5, "rtol": 1e-5,
+        "inputs": [{"name": "a", "shape": [256, 384], "dtype": "f32"}],
+        "outputs": [{"name": "c", "shape": [256, 384], "dtype": "f32", "tile": [32, 64]}]}))[0]
+    p = M.plan(entry, seed=4)
+    arena = torch.zeros(p.arena_bytes, dtype=torch.uint8, device=dev)
+    M.synthesize(p, arena)
+    a = arena[p.inputs["a"]: p.inputs["a"] + 4 * 256 * 384].view(torch.float32)
+    assert abs(a.mean().item() - 5.0) < 0.2 and abs(a.std().item() - 10.0) < 0.2  # N(5, 10)
+    n = 256 * 384
+    sv.generate([sv.GenSpec("f32", "from_arena", n, seed=4, stream=9, ref_offset=p.ref_outputs["c"],
+                            cand_offset=p.cand_outputs["c"], a_offset=p.inputs["a"],
+                            pcount=sv.Perturb("count_add", stream=3, count=2, value=1.0))], arena)
+    got = M.verify(p, arena)["c"]
+    t = p.tiles["c"]
+    bad = M.failing_tiles(got, t)
+    assert len(bad) in (1, 2) and sum(r["mismatches"] for r in got) == 2
+    for (ti, tj) in bad:
+        f = got[ti * 6 + tj]["first_mismatch"]
+        assert (f // 384 // 32, f % 384 // 64) == (ti, tj)
+    want = oracle.compare_tiles(t, arena.cpu().numpy(), arena.cpu().numpy())
+    assert_results_match(got, want, "manifest plan")
