@@ -168,3 +168,30 @@ def test_manifest_plan_end_to_end(dev):
         assert (f // 384 // 32, f % 384 // 64) == (ti, tj)
     want = oracle.compare_tiles(t, arena.cpu().numpy(), arena.cpu().numpy())
     assert_results_match(got, want, "manifest plan")
+
+
+def test_medium_output_per_tile(dev):
+    """An 8192 x 8192 bf16 output (2 x 128 MiB, beyond L2) in 64 x 64 tiles
+    (16384 verdicts, one warp per tile), with relative noise on the candidate;
+    sampled tile rows are recomputed by the oracle from the same bytes."""
+    import torch
+    side = 8192
+    ref = torch.randn(side * side, dtype=torch.float32, device=dev) * 10 + 5
+    cand = ref * (1 + torch.randn_like(ref) * 2 ** -9)
+    ref16, cand16 = ref.to(torch.bfloat16), cand.to(torch.bfloat16)
+    cand16[123456] = float("nan")
+    cand16[side * 4000 + 77] += 3.0
+    arena = torch.cat([cand16.view(torch.uint8), ref16.view(torch.uint8)])
+    t = W.Tiles("bf16", side, side, 0, 2 * side * side, tile_rows=64, tile_cols=64, atol=1e-2, rtol=1e-2)
+    got = sv.decode_results(sv.compare_tiles(t, arena, arena), 128 * 128)
+    for ti in (0, 62, 127):
+        lo, hi = 64 * ti * side * 2, 64 * (ti + 1) * side * 2
+        c = arena[lo:hi].cpu().numpy()
+        r = arena[2 * side * side + lo: 2 * side * side + hi].cpu().numpy()
+        want = oracle.compare_tiles(W.Tiles("bf16", 64, side, 0, 0, tile_rows=64, tile_cols=64, atol=1e-2,
+                                            rtol=1e-2), c, r)
+        for w in want:
+            if w["first_mismatch"] >= 0:
+                w["first_mismatch"] += 64 * ti * side
+        assert_results_match(got[128 * ti: 128 * ti + 128], want, "tile row %d" % ti)
+    assert sum(g["mismatches"] for g in got) >= 2 and got[62 * 128 + 1]["first_mismatch"] == side * 4000 + 77
