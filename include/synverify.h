@@ -279,7 +279,8 @@ int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, 
  * hundred tiles or more.  rows or cols 0: nothing to do.
  * Errors: SV_EINVAL (type, flags, tolerance, zero tile extent, pitch < cols,
  * a tile wider or taller than 2^31 - 1), SV_EALIGN, SV_ERANGE (operand beyond
- * its buffer, more than SV_MAX_TILES tiles), SV_ECUDA. */
+ * its buffer, more than SV_MAX_TILES tiles, a row pitch of 4 GiB or more
+ * when tiles span several rows), SV_ECUDA. */
 int verify_compare_tiles(const vc_tiles* tiles, const void* d_cand, size_t cand_bytes, const void* d_ref,
                          size_t ref_bytes, vc_result* d_results, sv_stream_t stream);
 

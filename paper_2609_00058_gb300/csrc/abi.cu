@@ -191,6 +191,8 @@ static int check_tiles(const vc_tiles& t, uint64_t cand_bytes, uint64_t ref_byte
   if (t.cand_offset % 16 || t.ref_offset % 16) return SV_EALIGN;
   if (t.rows > 1 && ((t.cand_pitch * sz) % 16 || (t.ref_pitch * sz) % 16)) return SV_EALIGN;
   if (t.tile_cols < t.cols && (t.tile_cols * sz) % 16) return SV_EALIGN;
+  // a tile that spans rows steps between them with 32-bit byte pitches
+  if (th > 1 && (t.cand_pitch * sz > 0xFFFFFFFFull || t.ref_pitch * sz > 0xFFFFFFFFull)) return SV_ERANGE;
   // the last element of each operand: offset + ((rows - 1) * pitch + cols) * size, without overflow
   for (int k = 0; k < 2; ++k) {
     const uint64_t pitch = k ? t.ref_pitch : t.cand_pitch, off = k ? t.ref_offset : t.cand_offset;

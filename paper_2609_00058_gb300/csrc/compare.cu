@@ -618,6 +618,11 @@ __global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant
     const uint32_t h = live ? (uint32_t)(umin(r0 + t.tile_rows, t.rows) - r0) : 0;
     const uint32_t w = live ? (uint32_t)(umin(c0 + t.tile_cols, t.cols) - c0) : 0;
     const uint32_t vr = w / VE;  // whole vectors per row of the tile
+    // the tile's origin in each operand; a row step is a 32 x 32 -> 64-bit
+    // multiply (row pitches under 4 GiB when a tile spans rows: validated)
+    const uint8_t* xt = xb + (r0 * t.cand_pitch + c0) * sz;
+    const uint8_t* yt = yb + (r0 * t.ref_pitch + c0) * sz;
+    const uint32_t xpb = (uint32_t)(t.cand_pitch * sz), ypb = (uint32_t)(t.ref_pitch * sz);
     Acc a;
     acc_reset(a);
     if (vr > 0) {
@@ -635,9 +640,9 @@ __global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant
 #pragma unroll
         for (int u = 0; u < U; ++u) {
           if (rr[u] < h) {
-            const uint64_t row = r0 + rr[u], col = c0 + (uint64_t)cc[u] * VE;
-            x[u] = ldg_stream(reinterpret_cast<const uint4*>(xb + (row * t.cand_pitch + col) * sz));
-            y[u] = ldg_stream(reinterpret_cast<const uint4*>(yb + (row * t.ref_pitch + col) * sz));
+            const uint32_t cb = cc[u] * 16u;
+            x[u] = ldg_stream(reinterpret_cast<const uint4*>(xt + (uint64_t)rr[u] * xpb + cb));
+            y[u] = ldg_stream(reinterpret_cast<const uint4*>(yt + (uint64_t)rr[u] * ypb + cb));
           }
         }
 #pragma unroll
