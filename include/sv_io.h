@@ -38,7 +38,7 @@
  * its copies and kernels; calls of one process are serialised by a lock.  The
  * library keeps SV_IO_SLOTS pinned host buffers of SV_IO_CHUNK_BYTES for file
  * data (allocated on first use, kept for the life of the process) and a pool
- * of host threads that read and write file stripes in parallel.  It allocates
+ * of host threads that read file stripes in parallel.  It allocates
  * no device memory: a conversion stages file bytes in the caller's workspace.
  */
 #ifndef SV_IO_H

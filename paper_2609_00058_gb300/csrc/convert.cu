@@ -194,7 +194,11 @@ template <Mode kMode, class S> __device__ __forceinline__ float to_f32(S x, uint
       const float r = __uint2float_rz((unsigned)x);
       return __uint_as_float(__float_as_uint(r) | (__float2uint_rz(r) != (unsigned)x ? 1u : 0u));
     }
-  } else {  // 64-bit integers and fp64: integer rounding
+  } else if constexpr (kMode == kNearestEven && (std::is_same<S, int64_t>::value ||
+                                                  std::is_same<S, uint64_t>::value)) {
+    // to nearest: the 64-bit integer conversion instruction
+    return std::is_same<S, int64_t>::value ? __ll2float_rn((long long)x) : __ull2float_rn((unsigned long long)x);
+  } else {  // 64-bit integers (to odd) and fp64: integer rounding
     if constexpr (std::is_same<S, double>::value) {
       // fast path, 32-bit steps: a result in fp32's normal range (biased fp64
       // exponent 897 ... 1150); the top 35 bits of the fp64 encoding less the

@@ -2,11 +2,13 @@
 // helpers (Sec. 4.1.2) made dtype-correct (Sec. 5.2.3).
 //
 // A file moves in chunks through SV_IO_SLOTS pinned host buffers.  A pool of
-// host threads reads (or writes) the stripes of one chunk in parallel while
-// the chunks before it cross the NVLink-C2C link with cudaMemcpyAsync and,
-// when the element types differ, are converted on the GPU (convert.cu) from a
-// two-chunk staging area in the caller's workspace.  A pinned buffer is
-// reused only after an event shows that the copy out of (or into) it is done.
+// host threads reads the stripes of one chunk in parallel while the chunks
+// before it cross the NVLink-C2C link with cudaMemcpyAsync and, when the
+// element types differ, are converted on the GPU (convert.cu) from a
+// two-chunk staging area in the caller's workspace.  Writes run the other
+// way, one writer thread per chunk while later chunks come back from the GPU.
+// A pinned buffer is reused only after an event shows that the copy out of
+// (or into) it is done.
 #include <cuda_runtime.h>
 #include <errno.h>
 #include <fcntl.h>
@@ -183,8 +185,11 @@ int pwrite_all(int fd, const uint8_t* src, uint64_t off, uint64_t len) {
   return SV_OK;
 }
 
-// one chunk's bytes moved by the pool in stripes of at least kStripeMin
+// one chunk's bytes moved by the pool in stripes of at least kStripeMin.
+// Writes take one thread: file systems serialise writers of one file (on the
+// GB300 hosts 1 and 16 pwrite threads reach the same rate).
 int parallel_io(bool write, int fd, uint8_t* buf, uint64_t off, uint64_t len) {
+  if (write) return pwrite_all(fd, buf, off, len);
   const uint64_t want = std::max<uint64_t>(1, len / kStripeMin);
   const int stripes = (int)std::min<uint64_t>(want, (uint64_t)pool().threads());
   const uint64_t stripe = ((len + stripes - 1) / stripes + 4095) / 4096 * 4096;
@@ -193,7 +198,7 @@ int parallel_io(bool write, int fd, uint8_t* buf, uint64_t off, uint64_t len) {
     const uint64_t b = (uint64_t)i * stripe;
     if (b >= len) return;
     const uint64_t l = std::min(stripe, len - b);
-    const int rc = write ? pwrite_all(fd, buf + b, off + b, l) : pread_all(fd, buf + b, off + b, l);
+    const int rc = pread_all(fd, buf + b, off + b, l);
     if (rc != SV_OK) err.store(rc);
   });
   return err.load();
