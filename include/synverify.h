@@ -257,6 +257,33 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
                    const void* d_ref, size_t ref_bytes, vc_result* d_results, void* d_ws, size_t ws_bytes,
                    sv_stream_t stream);
 
+/* A prepared verify_compare, for callers that compare many candidates on the
+ * same segments (every candidate of a round is checked on the same stage
+ * layout): the pair table is validated, grouped, scheduled and (beyond
+ * SV_INLINE_ENTRIES pairs) copied into the workspace once, so that each
+ * verify_compare_planned call only enqueues its launches.
+ *   sv_compare_plan_create: pairs as verify_compare, checked against buffers
+ *     of cand_bytes / ref_bytes; d_ws, ws_bytes >= sv_compare_workspace_bytes()
+ *     of the same table.  Synchronous: it returns once the table is in the
+ *     workspace.  *plan receives a host object owned by the caller.
+ *   verify_compare_planned: the verdicts of verify_compare with the plan's
+ *     pairs, on buffers of at least the sizes the plan was checked against
+ *     (the caller keeps that promise; the plan does not see the buffers'
+ *     sizes), asynchronous on `stream`.  The plan's workspace holds the table
+ *     and the partial records: calls with one plan whose work can overlap on
+ *     the GPU race, and nothing else may use the workspace while the plan
+ *     lives.  The plan belongs to the device that was current at its creation.
+ *   sv_compare_plan_destroy: frees the host object (NULL: nothing); the
+ *     workspace stays the caller's.
+ * Errors: as verify_compare (create: also SV_ERANGE when out of host memory);
+ * planned: SV_EINVAL (null plan or buffers), SV_ECUDA. */
+typedef struct sv_compare_plan sv_compare_plan;
+int sv_compare_plan_create(const vc_pair* pairs, int n_pairs, size_t cand_bytes, size_t ref_bytes, void* d_ws,
+                           size_t ws_bytes, sv_stream_t stream, sv_compare_plan** plan);
+int verify_compare_planned(const sv_compare_plan* plan, const void* d_cand, const void* d_ref, vc_result* d_results,
+                           sv_stream_t stream);
+void sv_compare_plan_destroy(sv_compare_plan* plan);
+
 /* verify_progressive: progressive multi-stage validation (CUDA-Harness
  * Sec. 4.2.2, fail-fast order).  Stages are compared in the given order
  * (size-ascending by convention); once a stage fails, every later stage is

@@ -181,6 +181,10 @@ EXPORTS = [
     ("sv_kernel_launches", C.c_uint64, []),
     ("syn_box_muller", C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
     ("sv_debug_fail_launches", C.c_int, [C.c_int]),
+    ("sv_compare_plan_create", C.c_int, [C.POINTER(vc_pair), C.c_int, _SZ, _SZ, _VP, _SZ, _VP,
+                                         C.POINTER(C.c_void_p)]),
+    ("verify_compare_planned", C.c_int, [_VP, _VP, _VP, _VP, _VP]),
+    ("sv_compare_plan_destroy", None, [_VP]),
     ("sv_check_tiles", C.c_int, [C.POINTER(vc_tiles), _SZ, _SZ, C.POINTER(C.c_uint64)]),
     ("verify_compare_tiles", C.c_int, [C.POINTER(vc_tiles), _VP, _SZ, _VP, _SZ, _VP, _VP]),
     # include/sv_io.h
@@ -321,6 +325,41 @@ def compare(pairs, cand, ref, results=None, workspace=None, stream=None):
                               results.data_ptr(), ws[0], ws[1] if ws[0] else 0, _stream_ptr(stream))
     _ok(rc, "verify_compare")
     return results
+
+
+class ComparePlan:
+    """sv_compare_plan_create: a verify_compare whose table is prepared once,
+    in a workspace this object owns, for buffers of cand_bytes / ref_bytes."""
+
+    def __init__(self, pairs, cand_bytes: int, ref_bytes: int, device=None, stream=None):
+        import torch
+        self.tab = pairs if isinstance(pairs, PairTable) else PairTable(pairs)
+        self.cand_bytes, self.ref_bytes = cand_bytes, ref_bytes
+        dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+        self._ws = _workspace(self.tab.ws_bytes, dev, None)
+        self._h = C.c_void_p()
+        rc = lib().sv_compare_plan_create(self.tab.arr, self.tab.n, cand_bytes, ref_bytes, self._ws[0],
+                                          self._ws[1] if self._ws[0] else 0, _stream_ptr(stream), C.byref(self._h))
+        _ok(rc, "sv_compare_plan_create")
+        self.n = self.tab.n
+        self.device = dev
+
+    def __call__(self, cand, ref, results=None, stream=None):
+        """verify_compare_planned; returns the device results tensor."""
+        import torch
+        if _nbytes(cand) < self.cand_bytes or _nbytes(ref) < self.ref_bytes:
+            raise ValueError("buffers smaller than the plan was made for")
+        if results is None:
+            results = torch.empty(max(self.n, 1) * RESULT_BYTES, dtype=torch.uint8, device=cand.device)
+        _ok(lib().verify_compare_planned(self._h, cand.data_ptr(), ref.data_ptr(), results.data_ptr(),
+                                         _stream_ptr(stream)), "verify_compare_planned")
+        return results
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h is not None and h.value and _lib is not None:
+            _lib.sv_compare_plan_destroy(h)
+            self._h = None
 
 
 def progressive(stages, cand, ref, results=None, first_failed=None, workspace=None, stream=None):

@@ -9,6 +9,7 @@
 #include <atomic>
 #include <cmath>
 #include <mutex>
+#include <new>
 #include <vector>
 
 #include "sv_device.cuh"
@@ -366,7 +367,84 @@ static bool ws_ok(const void* ws, size_t have, size_t need) {
   return ws && have >= need && reinterpret_cast<uintptr_t>(ws) % kAlign == 0;
 }
 
+// the plan of one verify_compare: the pair table grouped (many small segments
+// to one warp-per-segment launch, key kSmallKey; the rest one launch per
+// dtype), each group's launch shape, and every pair's units and partial slots
+constexpr uint32_t kSmallKey = 8;
+
+template <class Tab>
+static void build_pair_plan(const vc_pair* pairs, int n_pairs, Tab& tab, std::vector<Group>& groups) {
+  int n_small = 0;
+  for (int i = 0; i < n_pairs; ++i) n_small += cmp_vectors(pairs[i]) <= kSmallVectors;
+  const bool split = n_small >= kSmallMinPairs;
+  std::vector<int> order;
+  group_by(n_pairs, [&](int i) {
+    return split && cmp_vectors(pairs[i]) <= kSmallVectors ? kSmallKey : pairs[i].dtype;
+  }, order, groups);
+  uint64_t slot_base = 0;
+  for (Group& g : groups) {
+    if (g.key == kSmallKey) {  // one slot each; the combine reads just slot0
+      for (int k = g.begin; k < g.end; ++k) {
+        DevPair& d = tab[k];
+        d.p = pairs[order[k]];
+        d.work_begin = 0;
+        d.chunk = ~0ull >> 1;
+        d.slot0 = slot_base++;
+        d.orig = (uint32_t)order[k];
+        d.pad = 0;
+      }
+      continue;
+    }
+    for (int k = g.begin; k < g.end; ++k) {
+      g.tiles += cmp_tiles(pairs[order[k]]);
+      g.units += cmp_units(pairs[order[k]]);
+    }
+    g.sh = compare_shape(g.key, g.units, g.tiles);
+    uint64_t u = 0;
+    for (int k = g.begin; k < g.end; ++k) {
+      DevPair& d = tab[k];
+      d.p = pairs[order[k]];
+      d.work_begin = u;
+      d.chunk = g.sh.chunk;
+      d.slot0 = slot_base + (uint64_t)(k - g.begin);
+      d.orig = (uint32_t)order[k];
+      d.pad = 0;
+      u += cmp_units(d.p);
+    }
+    slot_base += g.sh.grid + (uint64_t)(g.end - g.begin) - 1;  // slots slot0 + b, b < grid
+  }
+}
+
+// the launches of a plan: one per group, then the combine
+static int run_pair_plan(const DevPair* host, const DevPair* dev, int n_pairs, const std::vector<Group>& groups,
+                         Partial* partials, const uint8_t* cand, const uint8_t* ref, vc_result* results,
+                         cudaStream_t st) {
+  for (const Group& g : groups) {
+    const DevPair* h = host + g.begin;
+    const DevPair* d = dev ? dev + g.begin : nullptr;
+    const cudaError_t e = g.key == kSmallKey
+                              ? launch_compare_small(h, d, g.end - g.begin, cand, ref, partials, st)
+                              : launch_compare_group(g.key, h, d, g.end - g.begin, g.units, g.sh, cand, ref, partials,
+                                                     nullptr, st);
+    if (e != cudaSuccess) return SV_ECUDA;
+  }
+  return status_of(launch_combine(host, dev, n_pairs, partials, results, nullptr, 0, st));
+}
+
 }  // namespace sv
+
+// a prepared verify_compare (synverify.h): the grouped table, kept on the host
+// for the launch parameters and, beyond SV_INLINE_ENTRIES pairs, in the
+// caller's workspace for the kernels
+struct sv_compare_plan {
+  int n = 0;
+  size_t cand_bytes = 0, ref_bytes = 0;
+  int device = -1;
+  std::vector<sv::DevPair> tab;
+  std::vector<sv::Group> groups;
+  const sv::DevPair* dev_tab = nullptr;
+  sv::Partial* partials = nullptr;
+};
 
 using namespace sv;
 
@@ -553,70 +631,64 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
   const size_t tb = pair_table_bytes(n_pairs);
   if (!ws_ok(d_ws, ws_bytes, tb + compare_partial_bytes(pairs, n_pairs))) return SV_EWORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  // many small segments go to one warp-per-segment launch (group key kSmallKey),
-  // the rest to one launch per dtype
-  constexpr uint32_t kSmallKey = 8;
-  int n_small = 0;
-  for (int i = 0; i < n_pairs; ++i) n_small += cmp_vectors(pairs[i]) <= kSmallVectors;
-  const bool split = n_small >= kSmallMinPairs;
-  std::vector<int> order;
   std::vector<Group> groups;
-  group_by(n_pairs, [&](int i) {
-    return split && cmp_vectors(pairs[i]) <= kSmallVectors ? kSmallKey : pairs[i].dtype;
-  }, order, groups);
   HostTable<DevPair> tab(n_pairs, tb != 0);
-  uint64_t slot_base = 0;
-  for (Group& g : groups) {
-    if (g.key == kSmallKey) {  // one slot each; the combine reads just slot0
-      for (int k = g.begin; k < g.end; ++k) {
-        DevPair& d = tab[k];
-        d.p = pairs[order[k]];
-        d.work_begin = 0;
-        d.chunk = ~0ull >> 1;
-        d.slot0 = slot_base++;
-        d.orig = (uint32_t)order[k];
-        d.pad = 0;
-      }
-      continue;
-    }
-    for (int k = g.begin; k < g.end; ++k) {
-      g.tiles += cmp_tiles(pairs[order[k]]);
-      g.units += cmp_units(pairs[order[k]]);
-    }
-    g.sh = compare_shape(g.key, g.units, g.tiles);
-    uint64_t u = 0;
-    for (int k = g.begin; k < g.end; ++k) {
-      DevPair& d = tab[k];
-      d.p = pairs[order[k]];
-      d.work_begin = u;
-      d.chunk = g.sh.chunk;
-      d.slot0 = slot_base + (uint64_t)(k - g.begin);
-      d.orig = (uint32_t)order[k];
-      d.pad = 0;
-      u += cmp_units(d.p);
-    }
-    slot_base += g.sh.grid + (uint64_t)(g.end - g.begin) - 1;  // slots slot0 + b, b < grid
-  }
+  build_pair_plan(pairs, n_pairs, tab, groups);
   uint8_t* ws = static_cast<uint8_t*>(d_ws);
   const DevPair* dev = nullptr;
   if (tb) {
     if (tab.upload(ws, st) != cudaSuccess) return SV_ECUDA;
     dev = reinterpret_cast<const DevPair*>(ws);
   }
-  Partial* partials = reinterpret_cast<Partial*>(ws + tb);
-  const uint8_t* cand = static_cast<const uint8_t*>(d_cand);
-  const uint8_t* ref = static_cast<const uint8_t*>(d_ref);
-  for (const Group& g : groups) {
-    const DevPair* h = tab.data() + g.begin;
-    const DevPair* d = dev ? dev + g.begin : nullptr;
-    const cudaError_t e = g.key == kSmallKey
-                              ? launch_compare_small(h, d, g.end - g.begin, cand, ref, partials, st)
-                              : launch_compare_group(g.key, h, d, g.end - g.begin, g.units, g.sh, cand, ref, partials,
-                                                     nullptr, st);
-    if (e != cudaSuccess) return SV_ECUDA;
-  }
-  return status_of(launch_combine(tab.data(), dev, n_pairs, partials, d_results, nullptr, 0, st));
+  return run_pair_plan(tab.data(), dev, n_pairs, groups, reinterpret_cast<Partial*>(ws + tb),
+                       static_cast<const uint8_t*>(d_cand), static_cast<const uint8_t*>(d_ref), d_results, st);
 }
+
+int sv_compare_plan_create(const vc_pair* pairs, int n_pairs, size_t cand_bytes, size_t ref_bytes, void* d_ws,
+                           size_t ws_bytes, sv_stream_t stream, sv_compare_plan** plan) {
+  if (!plan) return SV_EINVAL;
+  *plan = nullptr;
+  if (int rc = check_pairs(pairs, n_pairs, cand_bytes, ref_bytes)) return rc;
+  const size_t tb = pair_table_bytes(n_pairs);
+  if (n_pairs > 0 && !ws_ok(d_ws, ws_bytes, tb + compare_partial_bytes(pairs, n_pairs))) return SV_EWORKSPACE;
+  sv_compare_plan* p = new (std::nothrow) sv_compare_plan();
+  if (!p) return SV_ERANGE;
+  p->n = n_pairs;
+  p->cand_bytes = cand_bytes;
+  p->ref_bytes = ref_bytes;
+  if (cudaGetDevice(&p->device) != cudaSuccess) p->device = -1;
+  if (n_pairs > 0) {
+    p->tab.resize((size_t)n_pairs);
+    build_pair_plan(pairs, n_pairs, p->tab, p->groups);
+    uint8_t* ws = static_cast<uint8_t*>(d_ws);
+    p->partials = reinterpret_cast<Partial*>(ws + tb);
+    if (tb) {  // the table goes up once; the plan's launches read it from the workspace
+      cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+      if (cudaMemcpyAsync(ws, p->tab.data(), sizeof(DevPair) * (size_t)n_pairs, cudaMemcpyHostToDevice, st) !=
+              cudaSuccess ||
+          cudaStreamSynchronize(st) != cudaSuccess) {
+        cudaGetLastError();
+        delete p;
+        return SV_ECUDA;
+      }
+      p->dev_tab = reinterpret_cast<const DevPair*>(ws);
+    }
+  }
+  *plan = p;
+  return SV_OK;
+}
+
+int verify_compare_planned(const sv_compare_plan* plan, const void* d_cand, const void* d_ref, vc_result* d_results,
+                           sv_stream_t stream) {
+  if (!plan) return SV_EINVAL;
+  if (plan->n == 0) return SV_OK;
+  if (!d_results || (plan->cand_bytes && !d_cand) || (plan->ref_bytes && !d_ref)) return SV_EINVAL;
+  return run_pair_plan(plan->tab.data(), plan->dev_tab, plan->n, plan->groups, plan->partials,
+                       static_cast<const uint8_t*>(d_cand), static_cast<const uint8_t*>(d_ref), d_results,
+                       reinterpret_cast<cudaStream_t>(stream));
+}
+
+void sv_compare_plan_destroy(sv_compare_plan* plan) { delete plan; }
 
 int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, size_t cand_bytes,
                        const void* d_ref, size_t ref_bytes, vc_result* d_results, int32_t* d_first_failed,

@@ -239,3 +239,16 @@ def test_tile_counts(lib):
                          1 << 34, 1 << 34) == 1 << 30
     with pytest.raises(sv.SynVerifyError):
         sv.tile_count(_tiles(tile_cols=6))
+
+
+def test_compare_plan_refusals_before_any_copy(lib):
+    plan = C.c_void_p(123)
+    good = sv.PairTable([W.Pair("f32", 64, 0, 0, 1e-5, 1e-5)])
+    bad = sv.PairTable([W.Pair("f32", 64, 8, 0, 1e-5, 1e-5)])  # misaligned offset
+    assert lib.sv_compare_plan_create(bad.arr, 1, 4096, 4096, None, 0, None, C.byref(plan)) == -2
+    assert plan.value is None
+    many = sv.PairTable([W.Pair("f32", 64, 256 * i, 0, 1e-5, 1e-5) for i in range(9)])  # needs a table
+    assert lib.sv_compare_plan_create(many.arr, 9, 1 << 20, 4096, None, 0, None, C.byref(plan)) == -4
+    assert lib.sv_compare_plan_create(good.arr, 1, 4096, 4096, None, 0, None, None) == -1
+    assert lib.verify_compare_planned(None, None, None, None, None) == -1
+    lib.sv_compare_plan_destroy(None)  # nothing to free

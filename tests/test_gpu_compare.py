@@ -155,3 +155,21 @@ def test_repeated_calls_are_deterministic(dev):
     a = sv.decode_results(sv.compare([W.Pair("f32", n, 0, 0, 1e-3, 1e-3)], c, r), 1)[0]
     for _ in range(3):
         assert sv.decode_results(sv.compare([W.Pair("f32", n, 0, 0, 1e-3, 1e-3)], c, r), 1)[0] == a
+
+
+@pytest.mark.parametrize("n_pairs,seed", [(3, 11), (9, 12), (200, 13)])
+def test_compare_plan_matches_oracle_for_several_candidates(dev, n_pairs, seed):
+    """One plan, three candidates (the original and two edited copies): every
+    planned verdict equals the oracle's, and the unplanned call's."""
+    pairs, cand, ref = _segments(n_pairs, seed)
+    d_ref = to_dev(ref, dev)
+    plan = sv.ComparePlan(pairs, cand.size, ref.size, device=dev)
+    rng = np.random.default_rng(seed)
+    for k in range(3):
+        c = cand.copy()
+        if k:
+            c[rng.choice(c.size, 50, replace=False)] ^= np.uint8(1 << k)
+        d_c = to_dev(c, dev)
+        got = sv.decode_results(plan(d_c, d_ref), n_pairs)
+        assert_results_match(got, oracle.compare(pairs, c, ref), "plan candidate %d" % k)
+        assert_results_match(got, sv.decode_results(sv.compare(pairs, d_c, d_ref), n_pairs), "plan vs call")
