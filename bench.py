@@ -46,10 +46,10 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # a hash of the generator's sources they were taken on (None once they change)
 NCU_TRAFFIC = {
     # gen_kernel<f32, normal>, median of the 7 launches of one single-pass ncu launch
-    # list (profiles/launches_ladder.md): 122,880 B read + 1,312,933,120 B written; no
+    # list of the ladder step: 122,880 B read + 1,312,933,120 B written; no
     # fixup launch (the one exact-count edit is applied by the generating CTA)
     ("ladder", "c7ab7035e73bbe0a"): 1313085696,
-    # gen_kernel<i64, permutation>, median of 7 launches (profiles/launches_perm_i64.md):
+    # gen_kernel<i64, permutation>, median of 7 launches of the permutation step:
     # 2,013,440 B read + 4,231,760,384 B written; the 34 swap edits are fused
     ("perm_i64", "c7ab7035e73bbe0a"): 4233829888,
 }
