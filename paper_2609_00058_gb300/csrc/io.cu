@@ -186,8 +186,8 @@ int pwrite_all(int fd, const uint8_t* src, uint64_t off, uint64_t len) {
 }
 
 // one chunk's bytes moved by the pool in stripes of at least kStripeMin.
-// Writes take one thread: file systems serialise writers of one file (on the
-// GB300 hosts 1 and 16 pwrite threads reach the same rate).
+// Writes take one thread: file systems serialise writers of one file (one and
+// sixteen pwrite threads reached the same rate where this was measured).
 int parallel_io(bool write, int fd, uint8_t* buf, uint64_t off, uint64_t len) {
   if (write) return pwrite_all(fd, buf, off, len);
   const uint64_t want = std::max<uint64_t>(1, len / kStripeMin);
