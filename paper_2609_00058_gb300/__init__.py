@@ -456,6 +456,15 @@ def _path(path) -> bytes:
     return os.fsencode(os.fspath(path))
 
 
+def _dense_cuda(t, what: str):
+    """The library reads and writes n * size bytes from data_ptr(): only a
+    dense CUDA tensor describes that memory."""
+    if t.device.type != "cuda":
+        raise ValueError("%s must be a CUDA tensor (got %s)" % (what, t.device))
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous (a strided view would be read as dense memory)" % what)
+
+
 def tensor_probe(path) -> dict:
     """sv_tensor_probe: the checked header of a tensor file."""
     h = sv_tensor_header()
@@ -492,6 +501,7 @@ def read_tensor(path, dtype: Optional[str] = None, out=None, *, file_dtype: Opti
     if out is None:
         buf = torch.empty(max(n_file, 1) * IO_DTYPE_BYTES[dst], dtype=torch.uint8, device=dev)
     else:
+        _dense_cuda(out, "out")
         buf = out
     ws = _workspace(lib().sv_io_workspace_bytes(IO_DTYPES[src], IO_DTYPES[dst], n_file), dev, workspace)
     h = sv_tensor_header()
@@ -512,6 +522,7 @@ def write_tensor(path, src, dtype: Optional[str] = None, shape: Optional[Sequenc
                  stream=None) -> None:
     """sv_write_tensor: write a CUDA tensor's bytes to a tensor file (header
     with `dtype` and `shape`, default: the tensor's own)."""
+    _dense_cuda(src, "src")
     if dtype is None:
         names = {_torch_dtype(k): k for k in IO_DTYPES}
         dtype = names[src.dtype]
@@ -527,6 +538,9 @@ def convert(src, src_dtype: str, dst_dtype: str, n: Optional[int] = None, out=No
     """sv_convert: device-to-device value conversion; returns (out, lost),
     `lost` a device uint64 counter (added to, not reset, when given)."""
     import torch
+    _dense_cuda(src, "src")
+    if out is not None:
+        _dense_cuda(out, "out")
     if n is None:
         n = _nbytes(src) // IO_DTYPE_BYTES[src_dtype]
     if out is None:

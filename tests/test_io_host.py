@@ -172,3 +172,23 @@ def test_chunk_hook_arguments(lib):
     assert lib.sv_debug_io_chunk_bytes((32 << 20) + 4096) == -1
     assert lib.sv_debug_io_chunk_bytes(8192) == 0
     assert lib.sv_debug_io_chunk_bytes(0) == 0
+
+
+def test_binding_refuses_host_and_strided_tensors(lib, tmp_path):
+    """The binding passes data_ptr(): a host tensor or a strided view would be
+    taken for dense device memory, so both are refused before any call."""
+    torch = pytest.importorskip("torch")
+    host = torch.zeros(64, dtype=torch.float32)
+    with pytest.raises(ValueError, match="CUDA"):
+        sv.write_tensor(tmp_path / "h.svt", host)
+    with pytest.raises(ValueError, match="CUDA"):
+        sv.convert(host, "f32", "f64")
+    class FakeCuda:  # a strided view on a CUDA device, as far as the checks can tell
+        device = torch.device("cuda", 0)
+
+        def is_contiguous(self):
+            return False
+    with pytest.raises(ValueError, match="contiguous"):
+        sv.write_tensor(tmp_path / "s.svt", FakeCuda(), dtype="f32", shape=(8,))
+    with pytest.raises(ValueError, match="contiguous"):
+        sv.convert(FakeCuda(), "f32", "f64", n=8)
