@@ -291,6 +291,7 @@ def _workspace(nbytes: int, device, workspace):
     if nbytes == 0:
         return None, 0
     if workspace is not None:
+        _dense_cuda(workspace, "workspace")
         return workspace.data_ptr(), workspace.numel() * workspace.element_size()
     ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
     base = ws.data_ptr()
@@ -307,6 +308,7 @@ def _nbytes(t) -> int:
 # ---------------------------------------------------------------------------
 def generate(specs, arena, workspace=None, stream=None) -> None:
     """syn_generate into `arena` (a CUDA tensor; offsets are bytes into it)."""
+    _dense_cuda(arena, "arena")
     tab = specs if isinstance(specs, SpecTable) else SpecTable(specs)
     ws = _workspace(tab.ws_bytes, arena.device, workspace)
     rc = lib().syn_generate(tab.arr, tab.n, arena.data_ptr(), _nbytes(arena), ws[0], ws[1] if ws[0] else 0,
@@ -317,9 +319,12 @@ def generate(specs, arena, workspace=None, stream=None) -> None:
 def compare(pairs, cand, ref, results=None, workspace=None, stream=None):
     """verify_compare; returns the device results tensor (uint8, n x 80 bytes)."""
     import torch
+    _dense_cuda(cand, "cand")
+    _dense_cuda(ref, "ref")
     tab = pairs if isinstance(pairs, PairTable) else PairTable(pairs)
     if results is None:
         results = torch.empty(max(tab.n, 1) * RESULT_BYTES, dtype=torch.uint8, device=cand.device)
+    _dense_cuda(results, "results")
     ws = _workspace(tab.ws_bytes, cand.device, workspace)
     rc = lib().verify_compare(tab.arr, tab.n, cand.data_ptr(), _nbytes(cand), ref.data_ptr(), _nbytes(ref),
                               results.data_ptr(), ws[0], ws[1] if ws[0] else 0, _stream_ptr(stream))
@@ -347,10 +352,13 @@ class ComparePlan:
     def __call__(self, cand, ref, results=None, stream=None):
         """verify_compare_planned; returns the device results tensor."""
         import torch
+        _dense_cuda(cand, "cand")
+        _dense_cuda(ref, "ref")
         if _nbytes(cand) < self.cand_bytes or _nbytes(ref) < self.ref_bytes:
             raise ValueError("buffers smaller than the plan was made for")
         if results is None:
             results = torch.empty(max(self.n, 1) * RESULT_BYTES, dtype=torch.uint8, device=cand.device)
+        _dense_cuda(results, "results")
         _ok(lib().verify_compare_planned(self._h, cand.data_ptr(), ref.data_ptr(), results.data_ptr(),
                                          _stream_ptr(stream)), "verify_compare_planned")
         return results
@@ -365,11 +373,15 @@ class ComparePlan:
 def progressive(stages, cand, ref, results=None, first_failed=None, workspace=None, stream=None):
     """verify_progressive; returns (device results, device int32 first-failed index)."""
     import torch
+    _dense_cuda(cand, "cand")
+    _dense_cuda(ref, "ref")
     tab = stages if isinstance(stages, PairTable) else PairTable(stages, progressive=True)
     if results is None:
         results = torch.empty(max(tab.n, 1) * RESULT_BYTES, dtype=torch.uint8, device=cand.device)
     if first_failed is None:
         first_failed = torch.empty(1, dtype=torch.int32, device=cand.device)
+    _dense_cuda(results, "results")
+    _dense_cuda(first_failed, "first_failed")
     ws = _workspace(tab.ws_bytes, cand.device, workspace)
     rc = lib().verify_progressive(tab.arr, tab.n, cand.data_ptr(), _nbytes(cand), ref.data_ptr(), _nbytes(ref),
                                   results.data_ptr(), first_failed.data_ptr(), ws[0], ws[1] if ws[0] else 0,
@@ -395,10 +407,13 @@ def compare_tiles(tiles, cand, ref, results=None, stream=None):
     """verify_compare_tiles; returns the device results tensor (uint8, one
     80-byte vc_result per tile, row-major over the tile grid)."""
     import torch
+    _dense_cuda(cand, "cand")
+    _dense_cuda(ref, "ref")
     c = to_c_tiles(tiles)
     n = tile_count(tiles, _nbytes(cand), _nbytes(ref))
     if results is None:
         results = torch.empty(max(n, 1) * RESULT_BYTES, dtype=torch.uint8, device=cand.device)
+    _dense_cuda(results, "results")
     _ok(lib().verify_compare_tiles(C.byref(c), cand.data_ptr(), _nbytes(cand), ref.data_ptr(), _nbytes(ref),
                                    results.data_ptr(), _stream_ptr(stream)), "verify_compare_tiles")
     return results
@@ -408,9 +423,11 @@ def box_muller(words, out=None, stream=None):
     """syn_box_muller: the generator's Box-Muller step on a CUDA uint32 tensor
     of word pairs; returns (or fills) a float32 tensor of the same length."""
     import torch
+    _dense_cuda(words, "words")
     n_pairs = words.numel() // 2
     if out is None:
         out = torch.empty(2 * n_pairs, dtype=torch.float32, device=words.device)
+    _dense_cuda(out, "out")
     _ok(lib().syn_box_muller(words.data_ptr(), n_pairs, out.data_ptr(), _stream_ptr(stream)), "syn_box_muller")
     return out
 

@@ -362,6 +362,17 @@ static size_t compare_partial_bytes(const vc_pair* pairs, int n) {
 
 static int status_of(cudaError_t e) { return e == cudaSuccess ? SV_OK : SV_ECUDA; }
 
+// base addresses the kernels read and write with vector accesses: element
+// buffers 16-byte aligned (128-bit loads and stores at 16-byte offsets),
+// result records 8-byte aligned (64-bit fields), the ladder's flag 4-byte
+// aligned.  A misaligned base is refused before anything is enqueued, so a
+// byte view with an odd storage offset cannot fault the GPU.
+static bool misaligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) != 0; }
+static int check_bases(const void* cand, const void* ref, const void* results) {
+  if (misaligned(cand, 16) || misaligned(ref, 16) || misaligned(results, 8)) return SV_EALIGN;
+  return SV_OK;
+}
+
 static bool ws_ok(const void* ws, size_t have, size_t need) {
   if (need == 0) return true;
   return ws && have >= need && reinterpret_cast<uintptr_t>(ws) % kAlign == 0;
@@ -566,6 +577,7 @@ int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena
   if (int rc = check_specs(specs, n_specs, arena_bytes)) return rc;
   if (n_specs == 0) return SV_OK;
   if (!d_arena) return SV_EINVAL;
+  if (misaligned(d_arena, 16)) return SV_EALIGN;
   const size_t need = spec_table_bytes(n_specs);
   if (!ws_ok(d_ws, ws_bytes, need)) return SV_EWORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -628,6 +640,7 @@ int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t
   if (int rc = check_pairs(pairs, n_pairs, cand_bytes, ref_bytes)) return rc;
   if (n_pairs == 0) return SV_OK;
   if (!d_results || (cand_bytes && !d_cand) || (ref_bytes && !d_ref)) return SV_EINVAL;
+  if (int rc = check_bases(d_cand, d_ref, d_results)) return rc;
   const size_t tb = pair_table_bytes(n_pairs);
   if (!ws_ok(d_ws, ws_bytes, tb + compare_partial_bytes(pairs, n_pairs))) return SV_EWORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -683,6 +696,7 @@ int verify_compare_planned(const sv_compare_plan* plan, const void* d_cand, cons
   if (!plan) return SV_EINVAL;
   if (plan->n == 0) return SV_OK;
   if (!d_results || (plan->cand_bytes && !d_cand) || (plan->ref_bytes && !d_ref)) return SV_EINVAL;
+  if (int rc = check_bases(d_cand, d_ref, d_results)) return rc;
   return run_pair_plan(plan->tab.data(), plan->dev_tab, plan->n, plan->groups, plan->partials,
                        static_cast<const uint8_t*>(d_cand), static_cast<const uint8_t*>(d_ref), d_results,
                        reinterpret_cast<cudaStream_t>(stream));
@@ -696,6 +710,8 @@ int verify_progressive(const vc_pair* stages, int n_stages, const void* d_cand, 
   if (int rc = check_pairs(stages, n_stages, cand_bytes, ref_bytes)) return rc;
   if (!d_first_failed) return SV_EINVAL;
   if (n_stages > 0 && (!d_results || (cand_bytes && !d_cand) || (ref_bytes && !d_ref))) return SV_EINVAL;
+  if (misaligned(d_first_failed, 4)) return SV_EALIGN;
+  if (int rc = check_bases(d_cand, d_ref, d_results)) return rc;
   if (!ws_ok(d_ws, ws_bytes, sv_progressive_workspace_bytes(stages, n_stages))) return SV_EWORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   // the first group's combine sets the flag (failing stage or -1); an empty

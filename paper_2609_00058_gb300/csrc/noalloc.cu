@@ -85,6 +85,10 @@ extern "C" int verify_compare_noalloc(const vc_pair* pairs, int n_pairs, const v
   uint64_t slots = 0;
   for (const Run& r : runs) slots += std::min<uint64_t>(r.tiles, kGridCap) + (uint64_t)(r.end - r.begin);
   if (slots > SV_NOALLOC_SLOTS) return SV_ERANGE;
+  // 128-bit loads from the operands, 64-bit fields in the results: a
+  // misaligned base is refused here, before the scratch lookup or any launch
+  const uintptr_t operands = reinterpret_cast<uintptr_t>(d_cand) | reinterpret_cast<uintptr_t>(d_ref);
+  if ((operands & 15) || (reinterpret_cast<uintptr_t>(d_results) & 7)) return SV_EALIGN;
 
   Partial* scratch = nullptr;
   if (int rc = scratch_for_current_device(&scratch)) return rc;

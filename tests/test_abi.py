@@ -252,3 +252,71 @@ def test_compare_plan_refusals_before_any_copy(lib):
     assert lib.sv_compare_plan_create(good.arr, 1, 4096, 4096, None, 0, None, None) == -1
     assert lib.verify_compare_planned(None, None, None, None, None) == -1
     lib.sv_compare_plan_destroy(None)  # nothing to free
+
+
+def test_misaligned_base_pointers_rejected_before_any_launch(lib):
+    """Element buffers must start on 16 bytes and results on 8 (the kernels
+    move 128-bit vectors and 64-bit fields); a misaligned base -- a byte view
+    with an odd storage offset, say -- is refused with SV_EALIGN and nothing
+    is enqueued (these calls would otherwise launch)."""
+    tab = sv.PairTable([_pair()])
+    ws, wsb = 0x100000, 1 << 20
+    for cand, ref, res in ((0x1008, 0x2000, 0x3000), (0x1000, 0x2004, 0x3000), (0x1000, 0x2000, 0x3004)):
+        assert lib.verify_compare(tab.arr, 1, cand, 4096, ref, 4096, res, ws, wsb, None) == -2
+        assert lib.verify_compare_noalloc(tab.arr, 1, cand, 4096, ref, 4096, res, None) == -2
+    stages = sv.PairTable([_pair()], progressive=True)
+    assert lib.verify_progressive(stages.arr, 1, 0x1008, 4096, 0x2000, 4096, 0x3000, 0x5000, ws, wsb, None) == -2
+    assert lib.verify_progressive(stages.arr, 1, 0x1000, 4096, 0x2000, 4096, 0x3000, 0x5002, ws, wsb, None) == -2
+    spec = sv.SpecTable([_spec()])
+    assert lib.syn_generate(spec.arr, 1, 0x1008, 4096 * 4, None, 0, None) == -2
+    # a plan checks the buffers it is handed at every call
+    plan = C.c_void_p()
+    assert lib.sv_compare_plan_create(tab.arr, 1, 4096, 4096, ws, wsb, None, C.byref(plan)) == 0
+    try:
+        assert lib.verify_compare_planned(plan, 0x1000, 0x2008, 0x3000, None) == -2
+        assert lib.verify_compare_planned(plan, 0x1000, 0x2000, 0x3001, None) == -2
+    finally:
+        lib.sv_compare_plan_destroy(plan)
+
+
+def test_noalloc_slot_limit_boundary(lib):
+    """verify_compare_noalloc counts min(tiles, 4096) + pairs partial slots
+    per dtype against SV_NOALLOC_SLOTS = 4104.  A call landing exactly on
+    the limit passes the slot check (it then stops at the misaligned result
+    pointer, SV_EALIGN, before any launch); one slot more is SV_ERANGE."""
+    big, n = 1 << 40, 1 << 22  # 2^22 fp32 elements: 16 MiB, 1024 tiles of 16 KiB per pair
+    f32 = [W.Pair("f32", n, i << 24, i << 24) for i in range(8)]
+    bf16 = W.Pair("bf16", 16, 8 << 24, 8 << 24)  # one tile
+    # 8 f32 pairs: 8192 tiles -> 4096 + 8 = 4104 slots, exactly the limit
+    at_limit = sv.PairTable(f32)
+    assert lib.verify_compare_noalloc(at_limit.arr, 8, 0x1000, big, 0x1000, big, 0x2001, None) == -2
+    # 7 f32 pairs (4096 + 7) and one bf16 pair (1 + 1): 4105 slots, one too many
+    over = sv.PairTable(f32[:7] + [bf16])
+    assert lib.verify_compare_noalloc(over.arr, 8, 0x1000, big, 0x1000, big, 0x2001, None) == -3
+    # 6 f32 pairs (4096 + 6) and one bf16 pair (1 + 1): 4104 slots again
+    fits = sv.PairTable(f32[:6] + [bf16])
+    assert lib.verify_compare_noalloc(fits.arr, 7, 0x1000, big, 0x1000, big, 0x2001, None) == -2
+
+
+def test_binding_refuses_host_and_strided_tensors_before_any_launch():
+    """A CPU tensor's data_ptr() is a host address and a strided view is not
+    the dense memory the library reads: every binding call refuses both with
+    ValueError before it reaches the library."""
+    torch = pytest.importorskip("torch")
+    host = torch.zeros(4096, dtype=torch.uint8)
+    pairs = [_pair()]
+    with pytest.raises(ValueError, match="CUDA"):
+        sv.compare(pairs, host, host)
+    with pytest.raises(ValueError, match="CUDA"):
+        sv.progressive(pairs, host, host)
+    with pytest.raises(ValueError, match="CUDA"):
+        sv.generate([_spec()], torch.zeros(4096 * 4, dtype=torch.uint8))
+    with pytest.raises(ValueError, match="CUDA"):
+        sv.compare_tiles(_tiles(), host, host)
+    with pytest.raises(ValueError, match="CUDA"):
+        sv.box_muller(torch.zeros(8, dtype=torch.int32))
+    with pytest.raises(ValueError, match="CUDA"):
+        sv.convert(host, "u8", "f32")
+    strided = torch.zeros(8192, dtype=torch.uint8)[::2]
+    with pytest.raises(ValueError):
+        sv.compare(pairs, strided, strided)

@@ -1,12 +1,14 @@
-"""verify_compare_noalloc through the C ABI, against verify_compare.
+"""verify_compare_noalloc through the C ABI, against verify_compare and the
+CPU oracle.
 
 The allocation-free entry point serves callers that cannot allocate device
 memory (their process's GPU memory belongs to another component, or their
 path must not pay for an allocation): they pass only inputs and outputs and
 the library uses a fixed scratch array in its own device memory.  Its
 verdicts must equal those of verify_compare (which takes a caller
-workspace) within the tolerance the other parity tests use: every integer
-field and the max statistics exactly, RMS within 1e-6 relative.  Two calls in
+workspace) and those of the CPU oracle on the same bytes, within the
+tolerance the other parity tests use: every integer field and the max
+statistics exactly, RMS within 1e-6 relative.  Two calls in
 a row check that the shared scratch left by one call does not leak into the
 next.  This file is collected last so that a run stopping at the first
 failure has already run every other test; it also passes alone in a fresh
@@ -50,7 +52,7 @@ def _noalloc(pairs, dcand, dref, results, stream):
                                            dref.numel(), results.data_ptr(), stream)
 
 
-def test_noalloc_matches_workspace_compare_on_two_calls(dev):
+def test_noalloc_matches_workspace_compare_on_two_calls(dev, oracle):
     import torch
     stream = torch.cuda.current_stream().cuda_stream
     cases = [
@@ -64,7 +66,8 @@ def test_noalloc_matches_workspace_compare_on_two_calls(dev):
         results = torch.full((len(pairs) * sv.RESULT_BYTES,), 0xAB, dtype=torch.uint8, device=dev)
         assert _noalloc(pairs, dc, dr, results, stream) == 0
         got = sv.decode_results(results, len(pairs))
-        assert_results_match(got, want, "noalloc")
+        assert_results_match(got, want, "noalloc vs verify_compare")
+        assert_results_match(got, oracle.compare(pairs, cand, ref), "noalloc vs oracle")
     # and the same call twice on the same buffers
     pairs, cand, ref = cases[0]
     dc, dr = to_dev(cand, dev), to_dev(ref, dev)
