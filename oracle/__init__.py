@@ -17,10 +17,10 @@ import numpy as np
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 SRC = os.path.join(HERE, "oracle.c")
-SRCS = [SRC, os.path.join(HERE, "convert.c")]
+SRCS = [SRC, os.path.join(HERE, "convert.c"), os.path.join(HERE, "threads.c")]
 HDR = os.path.join(HERE, "oracle.h")
 LIB = os.path.join(HERE, "_build", "liboracle.so")
-CFLAGS = ["-O2", "-std=c11", "-Wall", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
+CFLAGS = ["-O2", "-std=c11", "-Wall", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared", "-pthread"]
 
 DTYPES = {"f32": 0, "f16": 1, "bf16": 2, "i32": 3, "i64": 4, "u32": 5}
 DTYPE_BYTES = {"f32": 4, "f16": 2, "bf16": 2, "i32": 4, "i64": 8, "u32": 4}
@@ -43,7 +43,7 @@ def build(force: bool = False) -> str:
     newest = max(os.path.getmtime(f) for f in SRCS + [HDR])
     if force or not os.path.exists(LIB) or os.path.getmtime(LIB) < newest:
         tmp = LIB + ".%d.tmp" % os.getpid()
-        subprocess.check_call(["gcc", *CFLAGS, "-o", tmp, *SRCS, "-lm"])
+        subprocess.check_call(["gcc", *CFLAGS, "-o", tmp, *SRCS, "-lm", "-lpthread"])
         os.replace(tmp, LIB)
     return LIB
 
@@ -127,6 +127,21 @@ def lib() -> C.CDLL:
         L.or_progressive.argtypes = [C.POINTER(PairC), C.c_int, C.c_void_p, C.c_uint64, C.c_void_p,
                                      C.c_uint64, C.POINTER(Result), C.POINTER(C.c_int32)]
         L.or_progressive.restype = C.c_int
+        L.or_compare_sums.argtypes = [C.POINTER(PairC), C.c_int, C.c_void_p, C.c_uint64, C.c_void_p,
+                                      C.c_uint64, C.POINTER(Result), C.POINTER(C.c_double)]
+        L.or_compare_sums.restype = C.c_int
+        L.or_check_pair.argtypes = [C.POINTER(PairC), C.c_uint64, C.c_uint64]
+        L.or_check_pair.restype = C.c_int
+        L.or_threads_default.argtypes = []
+        L.or_threads_default.restype = C.c_int
+        L.or_generate_mt.argtypes = [C.POINTER(Spec), C.c_int, C.c_void_p, C.c_uint64, C.c_int]
+        L.or_generate_mt.restype = C.c_int
+        L.or_compare_mt.argtypes = [C.POINTER(PairC), C.c_int, C.c_void_p, C.c_uint64, C.c_void_p, C.c_uint64,
+                                    C.POINTER(Result), C.c_int]
+        L.or_compare_mt.restype = C.c_int
+        L.or_progressive_mt.argtypes = [C.POINTER(PairC), C.c_int, C.c_void_p, C.c_uint64, C.c_void_p,
+                                        C.c_uint64, C.POINTER(Result), C.POINTER(C.c_int32), C.c_int]
+        L.or_progressive_mt.restype = C.c_int
         L.or_compare_tiles.argtypes = [C.POINTER(TilesC), C.c_void_p, C.c_uint64, C.c_void_p, C.c_uint64,
                                        C.POINTER(Result)]
         L.or_compare_tiles.restype = C.c_int
@@ -255,11 +270,21 @@ def check_spec(spec, arena_bytes: int) -> int:
     return lib().or_check_spec(C.byref(s), arena_bytes)
 
 
-def generate(specs, arena: np.ndarray) -> None:
-    """Run the specs in order into `arena` (uint8 numpy array, modified in place)."""
+def threads_default() -> int:
+    """Online host cores (the thread count of threads=0)."""
+    return lib().or_threads_default()
+
+
+def generate(specs, arena: np.ndarray, threads: int = 1) -> None:
+    """Run the specs into `arena` (uint8 numpy array, modified in place); the
+    specs of one call are independent.  threads != 1: the multi-threaded
+    driver (same bytes; 0 = every host core)."""
     assert arena.dtype == np.uint8 and arena.flags.c_contiguous
-    arr = (Spec * len(specs))(*[to_spec(s) for s in specs])
-    rc = lib().or_generate(arr, len(specs), arena.ctypes.data, arena.size)
+    arr = (Spec * max(len(specs), 1))(*[to_spec(s) for s in specs])
+    if threads == 1:
+        rc = lib().or_generate(arr, len(specs), arena.ctypes.data, arena.size)
+    else:
+        rc = lib().or_generate_mt(arr, len(specs), arena.ctypes.data, arena.size, threads)
     if rc != 0:
         raise ValueError("oracle: invalid generator spec")
 
@@ -269,36 +294,58 @@ def value_at(spec, arena: np.ndarray, g: int, role: int) -> int:
     return lib().or_value_at(C.byref(s), arena.ctypes.data, g, role)
 
 
-def compare(pairs, cand: np.ndarray, ref: np.ndarray) -> List[dict]:
-    arr = (PairC * len(pairs))(*[to_pair(p) for p in pairs])
-    out = (Result * len(pairs))()
-    rc = lib().or_compare(arr, len(pairs), cand.ctypes.data, cand.nbytes, ref.ctypes.data, ref.nbytes, out)
+def compare(pairs, cand: np.ndarray, ref: np.ndarray, threads: int = 1) -> List[dict]:
+    """Eq. 1 verdicts per pair; threads != 1: the multi-threaded driver
+    (integer fields identical, rms up to the order of its sum)."""
+    arr = (PairC * max(len(pairs), 1))(*[to_pair(p) for p in pairs])
+    out = (Result * max(len(pairs), 1))()
+    if threads == 1:
+        rc = lib().or_compare(arr, len(pairs), cand.ctypes.data, cand.nbytes, ref.ctypes.data, ref.nbytes, out)
+    else:
+        rc = lib().or_compare_mt(arr, len(pairs), cand.ctypes.data, cand.nbytes, ref.ctypes.data, ref.nbytes,
+                                 out, threads)
     if rc != 0:
         raise ValueError("oracle: invalid compare pair")
-    return [result_dict(r) for r in out]
+    return [result_dict(r) for r in out][:len(pairs)]
 
 
-def progressive(stages, cand: np.ndarray, ref: np.ndarray) -> Tuple[List[dict], int]:
-    arr = (PairC * len(stages))(*[to_pair(p) for p in stages])
-    out = (Result * len(stages))()
+def compare_sums(pairs, cand: np.ndarray, ref: np.ndarray) -> Tuple[List[dict], List[float]]:
+    """compare() plus each pair's sum of squared differences (index order)."""
+    arr = (PairC * max(len(pairs), 1))(*[to_pair(p) for p in pairs])
+    out = (Result * max(len(pairs), 1))()
+    sums = (C.c_double * max(len(pairs), 1))()
+    rc = lib().or_compare_sums(arr, len(pairs), cand.ctypes.data, cand.nbytes, ref.ctypes.data, ref.nbytes, out,
+                               sums)
+    if rc != 0:
+        raise ValueError("oracle: invalid compare pair")
+    return [result_dict(r) for r in out][:len(pairs)], list(sums)[:len(pairs)]
+
+
+def progressive(stages, cand: np.ndarray, ref: np.ndarray, threads: int = 1) -> Tuple[List[dict], int]:
+    arr = (PairC * max(len(stages), 1))(*[to_pair(p) for p in stages])
+    out = (Result * max(len(stages), 1))()
     ff = C.c_int32(0)
-    rc = lib().or_progressive(arr, len(stages), cand.ctypes.data, cand.nbytes, ref.ctypes.data, ref.nbytes,
-                              out, C.byref(ff))
+    if threads == 1:
+        rc = lib().or_progressive(arr, len(stages), cand.ctypes.data, cand.nbytes, ref.ctypes.data, ref.nbytes,
+                                  out, C.byref(ff))
+    else:
+        rc = lib().or_progressive_mt(arr, len(stages), cand.ctypes.data, cand.nbytes, ref.ctypes.data,
+                                     ref.nbytes, out, C.byref(ff), threads)
     if rc != 0:
         raise ValueError("oracle: invalid stage")
-    return [result_dict(r) for r in out], ff.value
+    return [result_dict(r) for r in out][:len(stages)], ff.value
 
 
-def run_workload(wl, arena: np.ndarray = None):
+def run_workload(wl, arena: np.ndarray = None, threads: int = 1):
     """Generate every call of a workload, then verify; returns (arena, results, first_failed)."""
     if arena is None:
         arena = np.zeros(wl.arena_bytes, dtype=np.uint8)
     for call in wl.gen_calls:
-        generate(call, arena)
+        generate(call, arena, threads=threads)
     if wl.progressive:
-        res, ff = progressive(wl.pairs, arena, arena)
+        res, ff = progressive(wl.pairs, arena, arena, threads=threads)
         return arena, res, ff
-    return arena, compare(wl.pairs, arena, arena), None
+    return arena, compare(wl.pairs, arena, arena, threads=threads), None
 
 
 def convert(src: np.ndarray, src_dtype: str, dst_dtype: str) -> Tuple[np.ndarray, int]:

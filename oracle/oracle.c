@@ -601,7 +601,14 @@ static int check_pair(const or_pair* p, uint64_t cand_bytes, uint64_t ref_bytes)
   return 0;
 }
 
-static void compare_one(const or_pair* p, const uint8_t* cand, const uint8_t* ref, or_result* r) {
+int or_check_pair(const or_pair* p, uint64_t cand_bytes, uint64_t ref_bytes) {
+  return check_pair(p, cand_bytes, ref_bytes);
+}
+
+/* one segment by the rule above; *sumsq_out receives the sum of squared     */
+/* differences behind r->rms (so chunked drivers can combine exact sums)     */
+static void compare_one_sum(const or_pair* p, const uint8_t* cand, const uint8_t* ref, or_result* r,
+                            double* sumsq_out) {
   memset(r, 0, sizeof(*r));
   r->first_mismatch = -1;
   r->state = OR_STAGE_RUN;
@@ -644,6 +651,7 @@ static void compare_one(const or_pair* p, const uint8_t* cand, const uint8_t* re
     r->max_abs = max_abs;
     r->max_rel = max_rel;
     r->rms = r->n_finite ? sqrt(sumsq / (double)r->n_finite) : 0.0;
+    *sumsq_out = sumsq;
   } else {
     double sumsq = 0.0, max_rel = 0.0;
     for (uint64_t i = 0; i < p->n; ++i) {
@@ -667,8 +675,14 @@ static void compare_one(const or_pair* p, const uint8_t* cand, const uint8_t* re
     r->max_abs = (double)r->max_abs_u64;
     r->max_rel = max_rel;
     r->rms = p->n ? sqrt(sumsq / (double)p->n) : 0.0;
+    *sumsq_out = sumsq;
   }
   r->pass = r->mismatches == 0;
+}
+
+static void compare_one(const or_pair* p, const uint8_t* cand, const uint8_t* ref, or_result* r) {
+  double sumsq;
+  compare_one_sum(p, cand, ref, r, &sumsq);
 }
 
 int or_compare(const or_pair* pairs, int n_pairs, const uint8_t* cand, uint64_t cand_bytes,
@@ -676,6 +690,14 @@ int or_compare(const or_pair* pairs, int n_pairs, const uint8_t* cand, uint64_t 
   for (int i = 0; i < n_pairs; ++i)
     if (check_pair(&pairs[i], cand_bytes, ref_bytes) != 0) return -1;
   for (int i = 0; i < n_pairs; ++i) compare_one(&pairs[i], cand, ref, &out[i]);
+  return 0;
+}
+
+int or_compare_sums(const or_pair* pairs, int n_pairs, const uint8_t* cand, uint64_t cand_bytes,
+                    const uint8_t* ref, uint64_t ref_bytes, or_result* out, double* sumsq) {
+  for (int i = 0; i < n_pairs; ++i)
+    if (check_pair(&pairs[i], cand_bytes, ref_bytes) != 0) return -1;
+  for (int i = 0; i < n_pairs; ++i) compare_one_sum(&pairs[i], cand, ref, &out[i], &sumsq[i]);
   return 0;
 }
 

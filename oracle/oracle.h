@@ -133,10 +133,35 @@ uint64_t or_value_at(const or_spec* s, const uint8_t* arena, uint64_t g, int rol
 int or_generate(const or_spec* specs, int n_specs, uint8_t* arena, uint64_t arena_bytes);
 
 /* ---- verification ---- */
+/* 0 if the pair is valid for buffers of these sizes, else -1 */
+int or_check_pair(const or_pair* p, uint64_t cand_bytes, uint64_t ref_bytes);
 int or_compare(const or_pair* pairs, int n_pairs, const uint8_t* cand, uint64_t cand_bytes,
                const uint8_t* ref, uint64_t ref_bytes, or_result* out);
 int or_progressive(const or_pair* stages, int n_stages, const uint8_t* cand, uint64_t cand_bytes,
                    const uint8_t* ref, uint64_t ref_bytes, or_result* out, int32_t* first_failed);
+/* or_compare that also returns each segment's sum of squared differences
+ * (the sum behind rms: rms = sqrt(sumsq / n_finite)), summed in index order */
+int or_compare_sums(const or_pair* pairs, int n_pairs, const uint8_t* cand, uint64_t cand_bytes,
+                    const uint8_t* ref, uint64_t ref_bytes, or_result* out, double* sumsq);
+
+/* ---- the same, spread over host threads (threads.c) ----
+ * For large inputs and for the CPU baseline measured on all host cores.
+ * Each spec or pair is cut into contiguous element chunks; every chunk runs
+ * through the single-threaded functions above (a spec chunk as a spec with
+ * its elem_offset and logical_n, a pair chunk as a pair at shifted offsets),
+ * and a pair's chunk verdicts are combined in chunk order: counts added,
+ * the first mismatch taken from the first chunk that has one, maxima
+ * maximised, sums of squares added.  Generated bytes and every integer
+ * field equal the single-threaded results exactly; rms differs only by the
+ * order of its fp64 sum.  nthreads <= 0: one thread per online host core.
+ * Returns as the single-threaded function. */
+int or_threads_default(void);
+int or_generate_mt(const or_spec* specs, int n_specs, uint8_t* arena, uint64_t arena_bytes, int nthreads);
+int or_compare_mt(const or_pair* pairs, int n_pairs, const uint8_t* cand, uint64_t cand_bytes,
+                  const uint8_t* ref, uint64_t ref_bytes, or_result* out, int nthreads);
+int or_progressive_mt(const or_pair* stages, int n_stages, const uint8_t* cand, uint64_t cand_bytes,
+                      const uint8_t* ref, uint64_t ref_bytes, or_result* out, int32_t* first_failed,
+                      int nthreads);
 
 /* ---- shaped outputs (Sec. 4.1.1: the manifest gives each output's shape) ----
  * A rows x cols output, row-major, with a row pitch (elements between row
