@@ -1,19 +1,29 @@
 """Benchmark of the synthesis + verification path on GB300.
 
-One step = the whole path over one batch: syn_generate of every stage's
-reference and candidate (test-data synthesis, CUDA-Harness Sec. 4.2.1) and
-verify_progressive over the stages (Eq. 1 and the fail-fast ladder,
-Sec. 4.2.2).  Default workload: the six-stage ladder n = 2^10 .. 2^27 fp32
-N(0,1) with 0.01% NaN/+-Inf/denormal injected, the candidate deviating at
-stage 4 (1.38 GB synthesized per step, 35.8 MB verified before the exit).
+One step = the whole path over one batch of one workload: syn_generate of
+every reference and candidate array (test-data synthesis, CUDA-Harness Sec.
+4.2.1), then the compare of every pair (Eq. 1) -- verify_progressive for the
+ladder (fail-fast, Sec. 4.2.2), a compare plan otherwise.
+
+Workloads (workloads.py): perm_i64 (int64 permutation n = 2^28, 17 swapped
+pairs; the default and headline: 4.29 GB synthesized and 4.29 GB verified
+per step), dotlike_bf16 (bf16 32768^2, K = 64), ladder (n = 2^10 .. 2^27
+fp32 N(0,1), exit at stage 3), segmented (4096 mixed-dtype cases) and
+fp32_pair (n = 2^20).  By default every workload is measured and the JSON
+line carries one object per workload under "workloads"; the top-level
+fields are the headline workload's.
 
 Prints ONE JSON line (rank 0).  `value` is synthesized + verified bytes per
 second with every buffer resident in HBM; `e2e` is the same metric through
 the public API with the synthesized test data delivered to pinned host
-memory and the verdicts read back every step.
+memory and the verdicts read back every step.  `roofline` is the headline
+workload's dominant kernel against the measured HBM copy bandwidth; the
+dot-like workload also reports its dot products' FMAs against a measured
+fp32 FMA rate (bench_alu_peak.cu).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--workload ladder|fp32_pair|segmented|dotlike_bf16|perm_i64|tensor_io]
+                  [--workload perm_i64|dotlike_bf16|ladder|segmented|fp32_pair|tensor_io]
+                  [--only-headline] [--no-cpu-baseline] [--oracle-threads T]
 
 --workload tensor_io measures the test-data I/O path instead (sv_read_tensor
 of a 1 GiB uint8 tensor file into fp32, the conversion kernel alone, the
@@ -42,17 +52,22 @@ import workloads as W  # noqa: E402
 METRIC = "verified GB/s and synthesized GB/s on 1 GB300, as % of HBM peak"
 L2_BYTES = 129 * 1000 * 1000  # GB300 L2 (bytes, nominal 129 MB)
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-# dram bytes per launch of the dominant kernel from one ncu capture, keyed by
-# a hash of the generator's sources they were taken on (None once they change)
+# DRAM bytes per step of each workload's generator and compare kernels from
+# one single-pass ncu launch list (dram__bytes_read.sum + dram__bytes_write.sum
+# summed over the step's launches of that role), keyed by (workload, role,
+# hash of the sources of that role's kernels): a figure taken on other
+# sources is not reported (null)
 NCU_TRAFFIC = {
-    # gen_kernel<f32, normal>, median of the 7 launches of one single-pass ncu launch
-    # list of the ladder step: 122,880 B read + 1,312,933,120 B written; no
-    # fixup launch (the one exact-count edit is applied by the generating CTA)
-    ("ladder", "c7ab7035e73bbe0a"): 1313085696,
-    # gen_kernel<i64, permutation>, median of 7 launches of the permutation step:
-    # 2,013,440 B read + 4,231,760,384 B written; the 34 swap edits are fused
-    ("perm_i64", "c7ab7035e73bbe0a"): 4233829888,
+    # gen_kernel<f32, normal>, median of the 7 launches of one launch list of
+    # the ladder step: 122,880 B read + 1,312,933,120 B written; the one
+    # exact-count edit is applied by the generating CTA (no fixup launch)
+    ("ladder", "generate", "c7ab7035e73bbe0a"): 1313085696,
+    # gen_kernel<i64, permutation>, median of 7 launches of the permutation
+    # step: 2,013,440 B read + 4,231,760,384 B written; the 34 swap edits fused
+    ("perm_i64", "generate", "c7ab7035e73bbe0a"): 4233829888,
 }
+ROLE_SOURCES = {"generate": ("generate.cu", "sv_device.cuh", "sv_kernels.h"),
+                "verify": ("compare.cu", "sv_device.cuh", "sv_kernels.h")}
 
 
 def log(*a):
@@ -69,56 +84,30 @@ def load_peaks():
 
 
 def alu_peaks():
-    """Philox blocks, Box-Muller pairs and fp32 FMAs per SM per cycle of the
-    library's own device code, measured now on this GPU by
-    paper_2609_00058_gb300/probes/alu_peak.cu (built on demand)."""
+    """Hardware issue rates (fp32 FMA, 32-bit IMAD, 32x32->64 IMAD per second
+    and per SM-cycle) measured now on this GPU by bench_alu_peak.cu, a plain
+    loop of independent chains of each instruction (built on demand)."""
     import subprocess
-    src = os.path.join(ROOT, "paper_2609_00058_gb300", "probes", "alu_peak.cu")
-    exe = os.path.join(ROOT, "paper_2609_00058_gb300", "_build", "alu_peak")
+    src = os.path.join(ROOT, "bench_alu_peak.cu")
+    exe = os.path.join(ROOT, "_build", "bench_alu_peak")
     try:
-        deps = [src] + [os.path.join(ROOT, "paper_2609_00058_gb300", "csrc", f) for f in ("sv_device.cuh", "sv_kernels.h")]
-        if not os.path.exists(exe) or os.path.getmtime(exe) < max(os.path.getmtime(d) for d in deps):
+        if not os.path.exists(exe) or os.path.getmtime(exe) < os.path.getmtime(src):
             from paper_2609_00058_gb300 import build as b
-            subprocess.run([b.nvcc(), *b.ARCH, "-O3", "-std=c++17", "--fmad=false", "-o", exe, src], check=True,
+            os.makedirs(os.path.dirname(exe), exist_ok=True)
+            subprocess.run([b.nvcc(), *b.ARCH, "-O3", "-std=c++17", "-o", exe, src], check=True,
                            capture_output=True, timeout=300)
         out = subprocess.run([exe], check=True, capture_output=True, text=True, timeout=120).stdout
         return json.loads(out.strip().splitlines()[-1])
-    except Exception as e:  # the roofline falls back to HBM alone
+    except Exception as e:  # the dot-like ALU fraction is then left out
         log("alu probe unavailable:", e)
         return None
 
 
-def alu_floor_s(wl, peaks):
-    """Seconds the generator needs at the measured ALU rates: per 4-element
-    quantum, its Philox blocks (value, special selection, element-wise
-    perturbation) and Box-Muller pairs (normal values, noise); for dot-like
-    values also the K fp32 FMAs of every output."""
-    cycles = 0.0
-    for call in wl.gen_calls:
-        for s in call:
-            quanta = (s.n + 3) // 4
-            if s.dist == "dotlike":  # K fp32 FMAs per output, then the same per-quantum noise
-                cycles += 4 * quanta * s.dot_k / peaks["ffma_per_sm_cycle"]
-                blocks = 1 if s.pelem.kind in ("rate_add_pm", "rel_noise") and s.cand_offset is not None else 0
-                pairs = 2 if s.pelem.kind == "rel_noise" else 0
-                cycles += quanta * (blocks / peaks["philox_blocks_per_sm_cycle"] +
-                                    pairs / peaks["box_muller_pairs_per_sm_cycle"])
-                continue
-            blocks = {"uniform": 1, "normal": 1, "int_range": 2 if s.dtype == "i64" else 1,
-                      "raw_bits": 2 if s.dtype == "i64" else 1}.get(s.dist, 0)
-            blocks += 1 if s.specials and s.special_rate > 0 else 0
-            blocks += 1 if s.pelem.kind in ("rate_add_pm", "rel_noise") and s.cand_offset is not None else 0
-            pairs = (2 if s.dist == "normal" else 0) + (2 if s.pelem.kind == "rel_noise" else 0)
-            cycles += quanta * (blocks / peaks["philox_blocks_per_sm_cycle"] +
-                                pairs / peaks["box_muller_pairs_per_sm_cycle"])
-    return cycles / (peaks["sms"] * peaks["clock_mhz"] * 1e6)
-
-
-def source_hash():
-    """Hash of the generator's kernel sources (the roofline's kernel)."""
+def source_hash(role):
+    """Hash of the kernel sources of one role ("generate" or "verify")."""
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2609_00058_gb300", "csrc")
-    for f in ("generate.cu", "sv_device.cuh", "sv_kernels.h"):
+    for f in ROLE_SOURCES[role]:
         with open(os.path.join(d, f), "rb") as fh:
             h.update(f.encode() + fh.read())
     return h.hexdigest()[:16]
@@ -201,59 +190,82 @@ def oracle_sample(workload):
     return W.int64_permutation_pair(1 << 22), "n=2^22 of the 2^28 permutation"
 
 
-def run_oracle_once(wl):
+def run_oracle_once(wl, threads=1):
+    """One step of the oracle on host memory: generate every call, then
+    verify; returns (seconds, synthesized + verified bytes)."""
     import oracle
     arena = np.zeros(wl.arena_bytes, np.uint8)
     t0 = time.perf_counter()
     for call in wl.gen_calls:
-        oracle.generate(call, arena)
+        oracle.generate(call, arena, threads=threads)
     if wl.progressive:
-        _, ff = oracle.progressive(wl.pairs, arena, arena)
+        _, ff = oracle.progressive(wl.pairs, arena, arena, threads=threads)
         stages = len(wl.pairs) if ff < 0 else ff + 1
     else:
-        oracle.compare(wl.pairs, arena, arena)
+        oracle.compare(wl.pairs, arena, arena, threads=threads)
         stages = None
     dt = time.perf_counter() - t0
     return dt, wl.synth_bytes() + wl.verify_bytes(stages)
 
 
-CPU_BASELINE_SECONDS = 10.0  # the sample is repeated until this much CPU work is timed
+CPU_BASELINE_SECONDS = 8.0  # per leg of the headline workload's baseline
+CPU_SUB_SECONDS = 2.0       # per leg of every other workload's baseline
 
 
-def cpu_baseline(workload):
-    wl, sample = oracle_sample(workload)
+def oracle_rate(wl, threads, seconds):
+    """GB/s of the oracle on `wl`, repeating it until `seconds` are timed."""
+    tot, nbytes, reps = 0.0, 0, 0
+    while reps == 0 or tot < seconds:
+        dt, nb = run_oracle_once(wl, threads)
+        tot, nbytes, reps = tot + dt, nbytes + nb, reps + 1
+    return nbytes / tot / 1e9, reps, tot
+
+
+def cpu_baseline(workload, seconds=CPU_BASELINE_SECONDS, threads=0):
+    """The oracle as it stands on a bounded sample of the workload, timed two
+    ways: single-threaded (the plain oracle) and on every host core (its
+    multi-threaded driver, same bytes and verdicts).  The top-level value is
+    the all-cores figure."""
     import oracle
     oracle.build()
-    tot, nbytes, reps = 0.0, 0, 0
-    while reps == 0 or tot < CPU_BASELINE_SECONDS:
-        dt, nb = run_oracle_once(wl)
-        tot, nbytes, reps = tot + dt, nbytes + nb, reps + 1
-    return {"value": nbytes / tot / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sample": "%d x (%s), generate + verify, single-threaded C oracle, %.1f s" % (reps, sample, tot)}
+    wl, sample = oracle_sample(workload)
+    cores = threads if threads > 0 else oracle.threads_default()
+    v1, r1, t1 = oracle_rate(wl, 1, seconds)
+    vt, rt, tt = oracle_rate(wl, cores, seconds)
+    single = {"value": v1, "unit": "GB/s", "cores": 1,
+              "sample": "%d x (%s), generate + verify, single-threaded C oracle, %.1f s" % (r1, sample, t1)}
+    threaded = {"value": vt, "unit": "GB/s", "cores": cores,
+                "sample": "%d x (%s), generate + verify, C oracle on %d threads, %.1f s" % (rt, sample, cores, tt)}
+    return {"value": vt, "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": threaded["sample"],
+            "single": single, "threaded": threaded}
 
 
 def reference_arm(args, rank, world):
+    """The oracle arm: the CPU oracle on all host cores (its multi-threaded
+    driver), one bounded sample of the workload per step."""
     if rank != 0:
         return
     import oracle
     oracle.build()
     if args.workload == "tensor_io":
         return io_reference_arm(args)
+    cores = args.oracle_threads if args.oracle_threads > 0 else oracle.threads_default()
     wl, sample = oracle_sample(args.workload)
     for _ in range(args.warmup):
-        run_oracle_once(wl)
+        run_oracle_once(wl, cores)
     times, nbytes = [], 0
     for _ in range(args.steps):
-        dt, nbytes = run_oracle_once(wl)
+        dt, nbytes = run_oracle_once(wl, cores)
         times.append(dt)
     tot = sum(times)
     value = nbytes * args.steps / tot / 1e9
+    what = "%s, C oracle on %d threads" % (sample, cores)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": workload_dtype(args.workload),
             "data": "synthetic (seeded counter-based specs)",
             "config": {"workload": full_workload(args.workload).name, "sample": sample},
-            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": what},
             "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -304,15 +316,36 @@ def workload_dtype(name):
             "perm_i64": "int64"}[name]
 
 
-def ours_arm(args, rank, world):
+WORKLOAD_ORDER = ("perm_i64", "dotlike_bf16", "ladder", "segmented", "fp32_pair")
+HEADLINE = "perm_i64"  # the largest single-GPU workload: 4.29 GB synthesized + 4.29 GB verified per step
+
+
+def timed_events(stream, fn, reps):
+    """Mean ms of fn() over reps calls, CUDA events on `stream` (after 3 warm-up calls)."""
+    import torch
+    for _ in range(3):
+        fn()
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    c0.record(stream)
+    for _ in range(reps):
+        fn()
+    c1.record(stream)
+    torch.cuda.synchronize()
+    return c0.elapsed_time(c1) / reps
+
+
+def measure_workload(name, args, dev, world, steps, warmup, alu):
+    """Time one workload's step (syn_generate, then the compare) with its
+    inputs resident in HBM, then the same step end to end through the
+    binding with the arena delivered to pinned host memory.  Returns the
+    workload's object of the JSON line (rank 0's view; times are max over
+    ranks)."""
     import torch
 
     import paper_2609_00058_gb300 as sv
 
-    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
-    torch.cuda.set_device(dev)
-    sv.lib()
-    wl = full_workload(args.workload)
+    wl = full_workload(name)
     arena = torch.zeros(wl.arena_bytes, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
     spec_tabs = [sv.SpecTable(c) for c in wl.gen_calls]
@@ -322,10 +355,9 @@ def ours_arm(args, rank, world):
     n_pairs = len(wl.pairs)
     results = torch.empty(n_pairs * sv.RESULT_BYTES, dtype=torch.uint8, device=dev)
     ff = torch.empty(1, dtype=torch.int32, device=dev)
-    synth_calls = [(t, c) for t, c in zip(spec_tabs, wl.gen_calls)]
 
     def do_generate():
-        for t, _ in synth_calls:
+        for t in spec_tabs:
             sv.generate(t, arena, workspace=ws)
 
     # a compare workload verifies through a plan built once (the pair table
@@ -349,7 +381,7 @@ def ours_arm(args, rank, world):
     synth_b, verify_b = wl.synth_bytes(), wl.verify_bytes(stages_run)
     step_bytes = synth_b + verify_b
 
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         do_generate()
         do_verify()
     torch.cuda.synchronize()
@@ -363,14 +395,14 @@ def ours_arm(args, rank, world):
     sampler = ClockSampler(dev)
     sampler.start()
     time.sleep(0.05)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier(world)
     torch.cuda.synchronize()
     launches0 = sv.lib().sv_kernel_launches()
     t_host0 = time.perf_counter()
     start.record(stream)
-    for k in range(args.steps):
+    for k in range(steps):
         if flush is not None:
             flush.fill_(k & 0xFF)
         ev[k][0].record(stream)
@@ -387,79 +419,77 @@ def ours_arm(args, rank, world):
     gen_each = [e[0].elapsed_time(e[1]) for e in ev]
     ver_each = [e[1].elapsed_time(e[2]) for e in ev]
     step_each = [g + v for g, v in zip(gen_each, ver_each)]
-    gen_ms = sum(gen_each) / args.steps
-    ver_ms = sum(ver_each) / args.steps
+    gen_ms = max_over_ranks(sum(gen_each) / steps, world)
+    ver_ms = max_over_ranks(sum(ver_each) / steps, world)
     # the job's time: start to end, or the sum of the steps when flushes sit between them
     total_ms = sum(step_each) if flush is not None else start.elapsed_time(end)
     total_ms = max_over_ranks(total_ms, world)
 
-    # the dot-like workload's candidate pass alone: the noisy twin of the
-    # existing reference array (SV_FROM_ARENA + relative noise), the part of
-    # its synthesis that is not the dot product
-    cand_pass = None
-    if args.workload == "dotlike_bf16":
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    reps = max(5, min(steps, 20))
+    extra = {}
+    if name == "dotlike_bf16":
+        # the candidate pass alone: the noisy twin of the existing reference
+        # array (SV_FROM_ARENA + relative noise), the part of its synthesis
+        # that is not the dot product
         d = wl.gen_calls[1][0]
         cp = sv.SpecTable([W.GenSpec(d.dtype, "from_arena", d.n, seed=d.seed, stream=d.stream, ref_offset=None,
                                      cand_offset=d.cand_offset, a_offset=d.ref_offset, pelem=d.pelem)])
-        for _ in range(3):
-            sv.generate(cp, arena, workspace=ws)
-        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        torch.cuda.synchronize()
-        c0.record(stream)
-        for _ in range(args.steps):
-            sv.generate(cp, arena, workspace=ws)
-        c1.record(stream)
-        torch.cuda.synchronize()
-        cp_ms = c0.elapsed_time(c1) / args.steps
+        cp_ms = timed_events(stream, lambda: sv.generate(cp, arena, workspace=ws), reps)
         cp_bytes = 2 * d.n * W.DTYPE_BYTES[d.dtype]  # reference read + candidate written
-        cand_pass = {"what": "candidate pass alone: reference read, noisy twin written", "ms": cp_ms,
-                     "bytes": cp_bytes, "gbs": cp_bytes / (cp_ms * 1e-3) / 1e9}
-
-    # the dot-like output compared per 128 x 128 tile (shaped outputs): the
-    # same bytes as the verify step, 65536 verdicts instead of one
-    tile_pass = None
-    if args.workload == "dotlike_bf16":
+        extra["candidate_pass"] = {"what": "candidate pass alone: reference read, noisy twin written", "ms": cp_ms,
+                                   "bytes": cp_bytes, "gbs": cp_bytes / (cp_ms * 1e-3) / 1e9,
+                                   "frac_of_hbm": cp_bytes / (cp_ms * 1e-3) / 1e9 / hbm}
+        # the dot products alone (factors in L2 or HBM, outputs written, no noise)
+        dot_only = sv.SpecTable([d.replace(cand_offset=None, pelem=W.Perturb())])
+        do_ms = timed_events(stream, lambda: sv.generate(dot_only, arena, workspace=ws), reps)
+        fmas = d.n * d.dot_k
+        extra["dot_only"] = {"what": "dot products alone: reference written, no candidate", "ms": do_ms,
+                             "fma_per_s": fmas / (do_ms * 1e-3)}
+        # the output compared per 128 x 128 tile (shaped outputs): the same
+        # bytes as the verify step, 65536 verdicts instead of one
         pr = wl.pairs[0]
         side = int(round(pr.n ** 0.5))
         tt = sv.Tiles(pr.dtype, side, side, pr.cand_offset, pr.ref_offset, tile_rows=128, tile_cols=128,
                       atol=pr.atol, rtol=pr.rtol)
         n_t = sv.tile_count(tt, wl.arena_bytes, wl.arena_bytes)
         tres = torch.empty(n_t * sv.RESULT_BYTES, dtype=torch.uint8, device=dev)
-        for _ in range(3):
-            sv.compare_tiles(tt, arena, arena, results=tres)
-        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        torch.cuda.synchronize()
-        c0.record(stream)
-        for _ in range(args.steps):
-            sv.compare_tiles(tt, arena, arena, results=tres)
-        c1.record(stream)
-        torch.cuda.synchronize()
-        tp_ms = c0.elapsed_time(c1) / args.steps
+        tp_ms = timed_events(stream, lambda: sv.compare_tiles(tt, arena, arena, results=tres), reps)
         tp_bytes = 2 * pr.n * W.DTYPE_BYTES[pr.dtype]
-        tile_pass = {"what": "verify_compare_tiles, %d x %d output in 128 x 128 tiles (%d verdicts)" % (side, side, n_t),
-                     "ms": tp_ms, "bytes": tp_bytes, "gbs": tp_bytes / (tp_ms * 1e-3) / 1e9}
+        extra["tile_verify"] = {"what": "verify_compare_tiles, %d x %d output in 128 x 128 tiles (%d verdicts)"
+                                        % (side, side, n_t), "ms": tp_ms, "bytes": tp_bytes,
+                                "gbs": tp_bytes / (tp_ms * 1e-3) / 1e9,
+                                "frac_of_hbm": tp_bytes / (tp_ms * 1e-3) / 1e9 / hbm}
+        if alu:
+            # the dot products' fp32 FMAs (K per output) against the measured
+            # FMA issue rate; the noise's Philox and Box-Muller work is not counted
+            peak = 2 * alu["ffma_per_s"] / 1e12
+            ach = 2 * fmas / (gen_ms * 1e-3) / 1e12
+            extra["alu"] = {"bound": "alu", "kernel": "dot_kernel<bf16> (syn_generate of the pair)",
+                            "achieved": ach, "peak": peak, "unit": "TFLOP/s", "frac": ach / peak,
+                            "dot_only_frac": 2 * fmas / (do_ms * 1e-3) / 1e12 / peak,
+                            "work": "%d outputs x K=%d fp32 FMAs (2 flops each); noise not counted" % (d.n, d.dot_k),
+                            "peak_kind": "measured fp32 FMA issue rate (bench_alu_peak.cu): %.1f FMA per SM-cycle "
+                                         "at %.0f MHz" % (alu["ffma_per_sm_cycle"], alu["ffma_mhz"])}
+        del tres
 
     # end to end: synthesized data delivered to pinned host buffers, verdicts read back
     host = torch.empty(wl.arena_bytes, dtype=torch.uint8, pin_memory=True)
     host_res = torch.empty(results.numel(), dtype=torch.uint8, pin_memory=True)
     host_ff = torch.empty(1, dtype=torch.int32, pin_memory=True)
-    # the whole arena (every output array and the few alignment gaps between
-    # them) goes back, in large pieces rather than one copy per array
-    out_ranges = [(0, wl.arena_bytes)]
     d2h = wl.arena_bytes + host_res.numel() + (4 if wl.progressive else 0)
-    h2d = sum(C.n * ctypes.sizeof(sv.syn_spec) for C in spec_tabs) + \
+    h2d = sum(t.n * ctypes.sizeof(sv.syn_spec) for t in spec_tabs) + \
         (pair_tab.n * ctypes.sizeof(sv.vc_pair) if wl.progressive else 0)  # a plan's table stays on the device
 
-    # the arena goes to pinned host memory in pieces of at most 64 MiB spread
-    # over four copy streams (several copy engines at once); the verify runs
-    # beside them on the compute stream, as both only read the arena
+    # the whole arena (every output array and the few alignment gaps between
+    # them) goes to pinned host memory in pieces of at most 64 MiB spread over
+    # four copy streams (several copy engines at once); the verify runs beside
+    # them on the compute stream, as both only read the arena
     copy_streams = [torch.cuda.Stream(dev) for _ in range(4)]
     pieces = [[] for _ in copy_streams]
-    k = 0
-    for off, nb in out_ranges:
-        for o in range(off, off + nb, 64 << 20):
-            pieces[k % len(pieces)].append((o, min(64 << 20, off + nb - o)))
-            k += 1
+    for k, o in enumerate(range(0, wl.arena_bytes, 64 << 20)):
+        pieces[k % len(pieces)].append((o, min(64 << 20, wl.arena_bytes - o)))
 
     def e2e_step():
         do_generate()
@@ -478,80 +508,127 @@ def ours_arm(args, rank, world):
             cs.synchronize()
         stream.synchronize()
 
-    e2e_steps = max(1, min(args.steps, 20))
-    for _ in range(min(args.warmup, 3)):
+    e2e_steps = max(1, min(steps, 20))
+    for _ in range(min(warmup, 3)):
         e2e_step()
     barrier(world)
     t0 = time.perf_counter()
     for _ in range(e2e_steps):
         e2e_step()
     e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+    del host, host_res, host_ff, arena, ws, results, flush, plan
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
 
-    if rank != 0:
-        return
-    peaks, peak_kind = load_peaks()
-    hbm = float(peaks["hbm_gbs"])
-    gen_bytes_launch = synth_b  # algorithmic bytes: every output element written once
-    achieved = gen_bytes_launch / (gen_ms * 1e-3) / 1e9
-    src = source_hash()
-    traffic = NCU_TRAFFIC.get((args.workload, src))
-    alu = alu_peaks()
-    alu_s = alu_floor_s(wl, alu) if alu else None
-    hbm_s = gen_bytes_launch / (hbm * 1e9)
-    if alu_s is not None and alu_s > hbm_s:
-        # the ALU floor is above the HBM floor: report against the output rate
-        # the measured Philox / Box-Muller throughput allows
-        alu_gbs = gen_bytes_launch / alu_s / 1e9
-        roofline = {"bound": "alu", "kernel": "syn_generate (gen_kernel + exact-count fixup)",
-                    "achieved": achieved, "peak": alu_gbs, "unit": "GB/s", "frac": achieved / alu_gbs,
-                    "peak_kind": "measured ALU rates (Philox %.3f blocks, Box-Muller %.3f pairs, %.1f fp32 FMAs "
-                                 "per SM-cycle, %d SMs at %d MHz) as output GB/s" % (
-                                     alu["philox_blocks_per_sm_cycle"], alu["box_muller_pairs_per_sm_cycle"],
-                                     alu["ffma_per_sm_cycle"], alu["sms"], alu["clock_mhz"]),
-                    "hbm_peak": hbm, "hbm_frac": achieved / hbm, "traffic": traffic}
-    else:
-        roofline = {"bound": "hbm", "kernel": "syn_generate (gen_kernel + exact-count fixup)",
-                    "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                    "peak_kind": "%s (%s)" % (peak_kind, "hbm_gbs"), "traffic": traffic}
-    line = {
-        "metric": METRIC,
-        "value": job_throughput(step_bytes, args.steps, world, total_ms * 1e-3),
-        "unit": "GB/s",
-        "n_gpus": world,
-        "steps": args.steps,
-        "warmup": args.warmup,
-        "ms_per_step": total_ms / args.steps,
-        "higher_is_better": True,
-        "scaling": "weak",
-        "vs_baseline": None,
-        "dtype": workload_dtype(args.workload),
-        "data": "synthetic (seeded counter-based specs)",
-        "config": {"workload": wl.name, "synth_bytes_per_step": synth_b, "verified_bytes_per_step": verify_b,
-                   "stages_run": stages_run,
-                   "l2": ("L2 flushed before every timed step (%d MiB written, outside the step's events)"
-                          % (2 * L2_BYTES >> 20)) if flush is not None else
-                         ("working set %.2f GB > 2 x 129 MB L2 per step (no flush)" % (wl.arena_bytes / 1e9)),
-                   "verify": "verify_progressive" if wl.progressive else
-                             "verify_compare_planned (plan built once, before the steps)",
-                   "parallelism": "replicas" if world > 1 else "single GPU"},
-        "synth_gbs": synth_b / (gen_ms * 1e-3) / 1e9,
-        "verify_gbs": verify_b / (ver_ms * 1e-3) / 1e9,
-        "synth_frac_of_hbm": synth_b / (gen_ms * 1e-3) / 1e9 / hbm,
-        "verify_frac_of_hbm": verify_b / (ver_ms * 1e-3) / 1e9 / hbm,
-        "gen_ms": gen_ms,
-        "verify_ms": ver_ms,
-        "step_ms_median": statistics.median(step_each),
-        "step_ms_best": min(step_each),
-        "roofline": roofline,
-        **({"candidate_pass": dict(cand_pass, frac_of_hbm=cand_pass["gbs"] / hbm)} if cand_pass else {}),
-        **({"tile_verify": dict(tile_pass, frac_of_hbm=tile_pass["gbs"] / hbm)} if tile_pass else {}),
+    gen_gbs = synth_b / (gen_ms * 1e-3) / 1e9
+    ver_gbs = verify_b / (ver_ms * 1e-3) / 1e9
+    gen_kernel = {"perm_i64": "gen_kernel<i64, permutation>", "ladder": "gen_kernel<f32, normal>",
+                  "dotlike_bf16": "dot_kernel<bf16>", "fp32_pair": "gen_kernel<f32, uniform>",
+                  "segmented": "gen_kernel<f32|f16|bf16 uniform, i32 int_range>"}[name]
+    cmp_kernel = "cmp_kernel<%s> + combine" % ("mixed" if name == "segmented" else wl.pairs[0].dtype)
+    out = {
+        "workload": wl.name,
+        "steps": steps, "warmup": warmup,
+        "synth_bytes_per_step": synth_b, "verified_bytes_per_step": verify_b, "stages_run": stages_run,
+        "l2": ("L2 flushed before every timed step (%d MiB written, outside the step's events)"
+               % (2 * L2_BYTES >> 20)) if flush is not None else
+              ("working set %.2f GB > 2 x 129 MB L2 per step (no flush)" % (wl.arena_bytes / 1e9)),
+        "verify": "verify_progressive" if wl.progressive else
+                  "verify_compare_planned (plan built once, before the steps)",
+        "value": job_throughput(step_bytes, steps, world, total_ms * 1e-3),
+        "ms_per_step": total_ms / steps,
+        "step_ms_median": statistics.median(step_each), "step_ms_best": min(step_each),
+        "gen_ms": gen_ms, "verify_ms": ver_ms,
+        "synth_gbs": gen_gbs, "verify_gbs": ver_gbs,
+        "synth_frac_of_hbm": gen_gbs / hbm, "verify_frac_of_hbm": ver_gbs / hbm,
+        "generate": {"kernel": gen_kernel, "ms": gen_ms, "bytes": synth_b, "gbs": gen_gbs, "frac_of_hbm": gen_gbs / hbm,
+                     "traffic": NCU_TRAFFIC.get((name, "generate", source_hash("generate")))},
+        "compare": {"kernel": cmp_kernel, "ms": ver_ms, "bytes": verify_b, "gbs": ver_gbs,
+                    "frac_of_hbm": ver_gbs / hbm, "traffic": NCU_TRAFFIC.get((name, "verify", source_hash("verify")))},
+        **extra,
         "e2e": {"value": job_throughput(step_bytes, e2e_steps, world, e2e_s), "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e2e_steps},
         "clocks": clocks,
         "gpu_launches": launches,
+        "hbm_peak": {"value": hbm, "unit": "GB/s", "kind": "%s (hbm_gbs)" % peak_kind},
     }
+    return out
+
+
+def roofline_of(sub):
+    """The dominant kernel of a workload's step against its bound: the
+    generator or the compare (whichever takes longer per step) against the
+    measured HBM copy bandwidth; the dot-like generator against the
+    measured fp32 FMA rate."""
+    dom = "generate" if sub["gen_ms"] >= sub["verify_ms"] else "compare"
+    if dom == "generate" and "alu" in sub:
+        r = dict(sub["alu"])
+        r["traffic"] = sub["generate"]["traffic"]
+        r["hbm_frac"] = sub["generate"]["frac_of_hbm"]
+        return r
+    k = sub[dom]
+    other = sub["compare" if dom == "generate" else "generate"]
+    return {"bound": "hbm", "kernel": k["kernel"], "achieved": k["gbs"], "peak": sub["hbm_peak"]["value"],
+            "unit": "GB/s", "frac": k["frac_of_hbm"], "traffic": k["traffic"],
+            "peak_kind": sub["hbm_peak"]["kind"],
+            "other_kernel": {"kernel": other["kernel"], "frac": other["frac_of_hbm"]}}
+
+
+def ours_arm(args, rank, world):
+    import torch
+
+    import paper_2609_00058_gb300 as sv
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    sv.lib()
+    headline = args.workload
+    names = [headline] + ([] if args.only_headline else [w for w in WORKLOAD_ORDER if w != headline])
+    alu = alu_peaks() if "dotlike_bf16" in names and rank == 0 else None
+    subs = {}
+    for name in names:
+        steps = args.steps if name == headline else min(args.steps, 20)
+        warmup = args.warmup if name == headline else max(3, min(args.warmup, 5))
+        log("measuring", name)
+        subs[name] = measure_workload(name, args, dev, world, steps, warmup, alu)
+    if rank != 0:
+        return
     if not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(args.workload)
+        for name in names:
+            subs[name]["cpu_baseline"] = cpu_baseline(
+                name, CPU_BASELINE_SECONDS if name == headline else CPU_SUB_SECONDS, args.oracle_threads)
+    h = subs[headline]
+    reasons = sorted({r for s in subs.values() for r in (s["clocks"].get("reasons") or [])})
+    line = {
+        "metric": METRIC,
+        "value": h["value"],
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": h["ms_per_step"],
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": workload_dtype(headline),
+        "data": "synthetic (seeded counter-based specs)",
+        "config": {"workload": h["workload"], "synth_bytes_per_step": h["synth_bytes_per_step"],
+                   "verified_bytes_per_step": h["verified_bytes_per_step"], "stages_run": h["stages_run"],
+                   "l2": h["l2"], "verify": h["verify"],
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "synth_gbs": h["synth_gbs"], "verify_gbs": h["verify_gbs"],
+        "synth_frac_of_hbm": h["synth_frac_of_hbm"], "verify_frac_of_hbm": h["verify_frac_of_hbm"],
+        "gen_ms": h["gen_ms"], "verify_ms": h["verify_ms"],
+        "roofline": roofline_of(h),
+        "e2e": h["e2e"],
+        "clocks": dict(h["clocks"], reasons_any_workload=reasons),
+        "gpu_launches": h["gpu_launches"],
+        "workloads": {n: dict(s, roofline=roofline_of(s)) for n, s in subs.items()},
+    }
+    if "cpu_baseline" in h:
+        line["cpu_baseline"] = h["cpu_baseline"]
+    if alu:
+        line["alu_peaks"] = alu
     print(json.dumps(line), flush=True)
 
 
@@ -732,8 +809,10 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="ladder", choices=sorted(W.FULL_SIZE) + ["tensor_io"])
+    ap.add_argument("--workload", default=HEADLINE, choices=sorted(W.FULL_SIZE) + ["tensor_io"])
+    ap.add_argument("--only-headline", action="store_true", help="measure the --workload alone")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--oracle-threads", type=int, default=0, help="oracle threads (0: every host core)")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

@@ -75,6 +75,10 @@ class RoundResult:
     first_failed: int  # index of the first failing stage, -1 if none (or not run)
     stages: List[dict] = field(default_factory=list)
     compile_log: str = ""
+    # with snapshot=True: (the compare pairs of the stages that ran, the
+    # arena's bytes on the host as they were verified), so the verdicts can
+    # be re-derived from the same data
+    snapshot: Optional[tuple] = None
 
 
 def reward(c: int, v: int, p: float) -> float:
@@ -153,8 +157,9 @@ def input_specs(task: Task, layout) -> List[GenSpec]:
 
 
 def run_round(task: Task, candidate_src: str, reference_src: str, work_dir: str, runs: int = 20,
-              flags: Sequence[str] = DEFAULT_FLAGS, device=None) -> RoundResult:
-    """Compile, synthesize, run, validate, time and score one candidate."""
+              flags: Sequence[str] = DEFAULT_FLAGS, device=None, snapshot: bool = False) -> RoundResult:
+    """Compile, synthesize, run, validate, time and score one candidate
+    (snapshot: also return the verified bytes, copied before the timing runs)."""
     import torch
     cand = compile_kernel(candidate_src, os.path.join(work_dir, "candidate"), flags)
     if not cand.ok:
@@ -189,9 +194,10 @@ def run_round(task: Task, candidate_src: str, reference_src: str, work_dir: str,
     res, ff = progressive(pairs, arena, arena, stream=stream)
     stages = decode_results(res, len(pairs))
     first_failed = int(ff.item())
+    snap = (pairs, arena.cpu().numpy()) if snapshot else None
     v = int(first_failed < 0)
     if not v:
-        return RoundResult(1, 0, 0.0, reward(1, 0, 0.0), None, first_failed, stages, cand.log)
+        return RoundResult(1, 0, 0.0, reward(1, 0, 0.0), None, first_failed, stages, cand.log, snap)
 
     # P of Eq. 3 on the largest stage: mean latency of `runs` launches (CUDA
     # events on the launching stream, after warm-up), reusing the candidate's
@@ -209,11 +215,11 @@ def run_round(task: Task, candidate_src: str, reference_src: str, work_dir: str,
     e1.synchronize()
     latency = e0.elapsed_time(e1) / runs
     p = 1.0 / latency
-    return RoundResult(1, 1, p, reward(1, 1, p), latency, -1, stages, cand.log)
+    return RoundResult(1, 1, p, reward(1, 1, p), latency, -1, stages, cand.log, snap)
 
 
 def run_program_round(task: Task, candidate_src: str, reference_src: str, work_dir: str, runs: int = 20,
-                      timeout: float = 120.0, device=None) -> RoundResult:
+                      timeout: float = 120.0, device=None, snapshot: bool = False) -> RoundResult:
     """One round with self-contained programs exchanging tensor files (the
     scaffold's process boundary, Sec. 4.1.2): the stage inputs are synthesized
     on the GPU and written to files; stage by stage, the reference and the
@@ -221,7 +227,8 @@ def run_program_round(task: Task, candidate_src: str, reference_src: str, work_d
     loaded back dtype-correctly (a file that is not float32 of the stage's
     size fails the stage) and compared with Eq. 1; the first failing stage
     ends the round (later stages are not run at all).  P is the candidate
-    program's mean latency over `runs` launches on the largest stage."""
+    program's mean latency over `runs` launches on the largest stage.
+    snapshot: also return the loaded outputs as they were compared."""
     import torch
     cand = compile_program(candidate_src, os.path.join(work_dir, "candidate"))
     if not cand.ok:
@@ -244,6 +251,7 @@ def run_program_round(task: Task, candidate_src: str, reference_src: str, work_d
                               timeout=timeout)
 
     stages: List[dict] = []
+    compared: List[Pair] = []
     first_failed = -1
     for s, (n, (a_off, b_off, r_off, c_off)) in enumerate(zip(task.stages, layout)):
         write_tensor(path("a", s), arena[a_off: a_off + 4 * n], dtype="f32", shape=(n,))
@@ -260,7 +268,9 @@ def run_program_round(task: Task, candidate_src: str, reference_src: str, work_d
             except SynVerifyError:
                 ok = False
         if ok:
-            res = decode_results(compare([Pair("f32", n, c_off, r_off, task.atol, task.rtol)], arena, arena), 1)[0]
+            pair = Pair("f32", n, c_off, r_off, task.atol, task.rtol)
+            compared.append(pair)
+            res = decode_results(compare([pair], arena, arena), 1)[0]
         else:
             res = {"state": 1, "pass": 0, "mismatches": n, "first_mismatch": 0, "max_abs": float("nan"),
                    "program_error": (cr.stderr or "").strip()[-500:]}
@@ -268,8 +278,9 @@ def run_program_round(task: Task, candidate_src: str, reference_src: str, work_d
         if not res["pass"]:
             first_failed = s
             break
+    snap = (compared, arena.cpu().numpy()) if snapshot else None
     if first_failed >= 0:
-        return RoundResult(1, 0, 0.0, reward(1, 0, 0.0), None, first_failed, stages, cand.log)
+        return RoundResult(1, 0, 0.0, reward(1, 0, 0.0), None, first_failed, stages, cand.log, snap)
     last = len(task.stages) - 1
     cr = run(cand.path, last, path("cand_t", last), (str(runs),))
     latency = None
@@ -277,9 +288,9 @@ def run_program_round(task: Task, candidate_src: str, reference_src: str, work_d
         if line.startswith("latency_ms "):
             latency = float(line.split()[1])
     if cr.returncode != 0 or latency is None or latency <= 0:
-        return RoundResult(1, 0, 0.0, reward(1, 0, 0.0), None, last, stages, cand.log)
+        return RoundResult(1, 0, 0.0, reward(1, 0, 0.0), None, last, stages, cand.log, snap)
     p = 1.0 / latency
-    return RoundResult(1, 1, p, reward(1, 1, p), latency, -1, stages, cand.log)
+    return RoundResult(1, 1, p, reward(1, 1, p), latency, -1, stages, cand.log, snap)
 
 
 def main(argv=None) -> int:

@@ -59,12 +59,28 @@ def test_broken_candidate_scores_minus_one(tmp_path):
     assert "scale_factor" in r.compile_log
 
 
+def assert_oracle_verdicts(r, progressive=True):
+    """The round's per-stage verdicts against the oracle on the bytes the
+    round verified (Eq. 1 per stage; Sec. 4.2.2 fail-fast for the ladder)."""
+    import oracle
+    from gpu_util import assert_results_match
+    pairs, h = r.snapshot
+    if progressive:
+        want, ff = oracle.progressive(pairs, h, h)
+        assert ff == r.first_failed
+    else:
+        want = oracle.compare(pairs, h, h)
+    assert_results_match(r.stages[:len(want)], want, "candidate round")
+    return want
+
+
 @pytest.mark.gpu
 def test_correct_candidate_round(tmp_path):
     from gpu_util import device
     device()
-    r = cr.run_round(TASK, src("vec_add_inplace"), src("vec_add_reference"), str(tmp_path))
+    r = cr.run_round(TASK, src("vec_add_inplace"), src("vec_add_reference"), str(tmp_path), snapshot=True)
     assert (r.C, r.V, r.first_failed) == (1, 1, -1)
+    assert_oracle_verdicts(r)
     assert r.latency_ms > 0 and r.P == pytest.approx(1.0 / r.latency_ms) and r.r == r.P
     assert all(s["state"] == sv.STAGE_RUN and s["pass"] and s["mismatches"] == 0 for s in r.stages)
     # the synthesized a carries NaN/Inf at the specials rate: both sides agree on them
@@ -76,14 +92,13 @@ def test_correct_candidate_round(tmp_path):
 def test_faulty_candidate_fails_at_the_first_large_stage(tmp_path):
     from gpu_util import device
     device()
-    r = cr.run_round(TASK, src("vec_add_inplace_faulty"), src("vec_add_reference"), str(tmp_path))
+    r = cr.run_round(TASK, src("vec_add_inplace_faulty"), src("vec_add_reference"), str(tmp_path), snapshot=True)
     assert (r.C, r.V, r.r, r.first_failed) == (1, 0, 0.0, 3)
     assert [s["state"] for s in r.stages] == [sv.STAGE_RUN] * 4
     assert [s["pass"] for s in r.stages] == [True, True, True, False]
-    # every element at or beyond 2^20 whose a * b is not negligible differs
-    bad = r.stages[3]
-    assert bad["first_mismatch"] >= 1 << 20
-    assert bad["mismatches"] > (TASK.stages[3] - (1 << 20)) // 2
+    # every statistic of every stage equals the oracle's on the same bytes
+    want = assert_oracle_verdicts(r)
+    assert want[3]["first_mismatch"] >= 1 << 20
 
 
 @pytest.mark.gpu
@@ -91,10 +106,11 @@ def test_fault_found_at_the_right_stage_on_other_ladders(tmp_path):
     from gpu_util import device
     device()
     task = cr.Task("vecAddInplace", stages=(1000, (1 << 20) - 1, (1 << 20) + 1, 1 << 21), seed=9)
-    r = cr.run_round(task, src("vec_add_inplace_faulty"), src("vec_add_reference"), str(tmp_path))
+    r = cr.run_round(task, src("vec_add_inplace_faulty"), src("vec_add_reference"), str(tmp_path), snapshot=True)
     assert r.first_failed == 2
     assert [s["state"] for s in r.stages] == [sv.STAGE_RUN] * 3 + [sv.STAGE_SKIPPED]
-    assert r.stages[2]["mismatches"] <= 1 and r.stages[2]["first_mismatch"] in (-1, 1 << 20)
+    assert_oracle_verdicts(r)
+    assert r.stages[2]["mismatches"] == 1 and r.stages[2]["first_mismatch"] == 1 << 20
 
 
 # ---------------------------------------------------------------------------
@@ -109,8 +125,9 @@ def test_broken_program_scores_minus_one(tmp_path):
 def test_correct_program_round(tmp_path):
     from gpu_util import device
     device()
-    r = cr.run_program_round(TASK, src("vec_add_inplace"), src("vec_add_reference"), str(tmp_path))
+    r = cr.run_program_round(TASK, src("vec_add_inplace"), src("vec_add_reference"), str(tmp_path), snapshot=True)
     assert (r.C, r.V, r.first_failed) == (1, 1, -1)
+    assert_oracle_verdicts(r, progressive=False)
     assert r.latency_ms > 0 and r.r == r.P == pytest.approx(1.0 / r.latency_ms)
     assert len(r.stages) == len(TASK.stages) and all(s["pass"] and s["mismatches"] == 0 for s in r.stages)
     # the files the programs exchanged are tensor files of the stage sizes
@@ -125,8 +142,10 @@ def test_faulty_program_stops_at_the_failing_stage(tmp_path):
     from gpu_util import device
     device()
     task = cr.Task("vecAddInplace", stages=(1000, 1 << 16, 1 << 21, 1 << 22), seed=3)
-    r = cr.run_program_round(task, src("vec_add_inplace_faulty"), src("vec_add_reference"), str(tmp_path))
+    r = cr.run_program_round(task, src("vec_add_inplace_faulty"), src("vec_add_reference"), str(tmp_path),
+                             snapshot=True)
     assert (r.C, r.V, r.r, r.first_failed) == (1, 0, 0.0, 2)
+    assert_oracle_verdicts(r, progressive=False)
     assert [s["pass"] for s in r.stages] == [True, True, False]
     assert r.stages[2]["first_mismatch"] >= 1 << 20
     assert not os.path.exists(os.path.join(str(tmp_path), "files", "a_3.svt"))

@@ -43,6 +43,15 @@ def _u(dtype):
     return {2: np.uint16, 4: np.uint32, 8: np.uint64}[W.DTYPE_BYTES[dtype]]
 
 
+def oracle_verdicts_on(arena_dev, wl):
+    """The oracle's verdicts on the GPU's own synthesized bytes (the arena
+    copied to the host), through its multi-threaded driver on every core."""
+    h = arena_dev.cpu().numpy()
+    if wl.progressive:
+        return oracle.progressive(wl.pairs, h, h, threads=0)
+    return oracle.compare(wl.pairs, h, h, threads=0), None
+
+
 def sample_indices(n, k, seed):
     rng = np.random.default_rng(seed)
     idx = set(rng.integers(0, n, size=k).tolist())
@@ -100,6 +109,10 @@ def test_ladder_full(dev):
     assert [g["mismatches"] for g in got[:4]] == [0, 0, 0, 1]
     s3 = wl.gen_calls[0][3]
     assert got[3]["first_mismatch"] == oracle.stratum_index(s3.n, 1, s3.seed, s3.pcount.stream, 0)
+    # the oracle's verdicts on the GPU's own bytes
+    want_g, want_gff = oracle_verdicts_on(arena, wl)
+    assert want_gff == 3
+    assert_results_match(got, want_g, "ladder, GPU bytes")
     # sampled synthesis of every stage, including the 2^25 and 2^27 ones
     h0 = np.zeros(16, np.uint8)
     for k, s in enumerate(wl.gen_calls[0]):
@@ -131,6 +144,8 @@ def test_dotlike_full(dev):
     import torch
     wl = W.dotlike_bf16_pair()
     arena, (got, _) = gpu_run(wl, dev)
+    # the verdict on the synthesized 2^30 pair equals the oracle's on the same bytes
+    assert_results_match(got, oracle_verdicts_on(arena, wl)[0], "dot-like, GPU bytes")
     fa, fb = wl.gen_calls[0]
     d = wl.gen_calls[1][0]
     # the oracle's own factors (2M normals each), uploaded in place of the
@@ -161,6 +176,10 @@ def test_perm_full(dev):
     import torch
     wl = W.int64_permutation_pair()
     arena, (got, _) = gpu_run(wl, dev)
+    # the verdict on the synthesized 2^28 pair equals the oracle's on the same bytes
+    want_g = oracle_verdicts_on(arena, wl)[0]
+    assert_results_match(got, want_g, "permutation, GPU bytes")
+    assert want_g[0]["mismatches"] <= 34
     s = wl.gen_calls[0][0]
     idx = sample_indices(s.n, 20000, 9)
     strata = [oracle.stratum_index(s.n, 34, s.seed, s.pcount.stream, k) for k in range(34)]
