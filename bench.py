@@ -516,6 +516,9 @@ def measure_workload(name, args, dev, world, steps, warmup, alu):
     for _ in range(e2e_steps):
         e2e_step()
     e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+    l2_note = ("L2 flushed before every timed step (%d MiB written, outside the step's events)"
+               % (2 * L2_BYTES >> 20)) if flush is not None else \
+        ("working set %.2f GB > 2 x 129 MB L2 per step (no flush)" % (wl.arena_bytes / 1e9))
     del host, host_res, host_ff, arena, ws, results, flush, plan
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
@@ -530,9 +533,7 @@ def measure_workload(name, args, dev, world, steps, warmup, alu):
         "workload": wl.name,
         "steps": steps, "warmup": warmup,
         "synth_bytes_per_step": synth_b, "verified_bytes_per_step": verify_b, "stages_run": stages_run,
-        "l2": ("L2 flushed before every timed step (%d MiB written, outside the step's events)"
-               % (2 * L2_BYTES >> 20)) if flush is not None else
-              ("working set %.2f GB > 2 x 129 MB L2 per step (no flush)" % (wl.arena_bytes / 1e9)),
+        "l2": l2_note,
         "verify": "verify_progressive" if wl.progressive else
                   "verify_compare_planned (plan built once, before the steps)",
         "value": job_throughput(step_bytes, steps, world, total_ms * 1e-3),

@@ -84,17 +84,28 @@ enum {
 };
 
 /* ---- special values (syn_spec.special_mask, OR of these) ----
- * Element g is special iff its SPECIAL_SEL word is < floor(rate * 2^32); its
- * kind is the j-th set bit of the mask (ascending), j = mulhi(w0, #kinds),
- * from SPECIAL_KIND block g.  NaN is the canonical quiet NaN; DENORM has a
- * random sign and a random nonzero fraction; DUP copies the base value of a
- * uniformly drawn index of the logical array.  Float types take NAN, PINF,
- * NINF, DENORM, ZERO, DUP; integer types ZERO, IMIN, IMAX, DUP. */
+ * Selection, Bernoulli mode (SV_SP_EXACT clear): element g is special iff
+ * its SPECIAL_SEL word is < floor(rate * 2^32).  Exact mode (SV_SP_EXACT
+ * set): exactly k = round(rate * N) elements of the logical array of N
+ * elements are special (k <= SV_MAX_COUNT, else SV_ERANGE), one per stratum
+ * of [0, N) cut into k equal strata, at floor(s N / k) + mulhi64(x, len) for
+ * stratum s, x = the first two words of SPECIAL_SEL block s.  The exact mode
+ * draws nothing per element, so a generator pass costs one Philox block less
+ * per 4-element quantum (a reading of "0.01% injected" as a count; the paper
+ * only asks for broad, special-laden inputs, Sec. 4.2.1).
+ * Kind, in both modes: the j-th set kind bit of the mask (ascending), j =
+ * mulhi(w0, #kinds), from SPECIAL_KIND block g.  NaN is the canonical quiet
+ * NaN; DENORM has a random sign and a random nonzero fraction; DUP copies the
+ * base value of a uniformly drawn index of the logical array.  Float types
+ * take NAN, PINF, NINF, DENORM, ZERO, DUP; integer types ZERO, IMIN, IMAX,
+ * DUP.  A mask with no kind bit selects nothing. */
 enum {
   SV_SP_NAN = 1u << 0, SV_SP_PINF = 1u << 1, SV_SP_NINF = 1u << 2,
   SV_SP_DENORM = 1u << 3, SV_SP_ZERO = 1u << 4, SV_SP_IMIN = 1u << 5,
   SV_SP_IMAX = 1u << 6, SV_SP_DUP = 1u << 7
 };
+#define SV_SP_KINDS 0xFFu
+#define SV_SP_EXACT (1u << 31)
 
 /* ---- candidate perturbations ----
  * Element-wise kinds (syn_spec.pelem):

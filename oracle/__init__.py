@@ -27,6 +27,7 @@ DTYPE_BYTES = {"f32": 4, "f16": 2, "bf16": 2, "i32": 4, "i64": 8, "u32": 4}
 DISTS = {"uniform": 0, "normal": 1, "int_range": 2, "permutation": 3, "dotlike": 4, "raw_bits": 5,
          "constant": 6, "from_arena": 7}
 SPECIALS = {"nan": 1, "pinf": 2, "ninf": 4, "denorm": 8, "zero": 16, "imin": 32, "imax": 64, "dup": 128}
+SPECIAL_EXACT = 1 << 31
 PERTS = {"none": 0, "rate_add_pm": 1, "rel_noise": 2, "count_set": 3, "count_add": 4, "swap_pairs": 5}
 PURPOSES = {"value": 0, "special_sel": 1, "special_kind": 2, "pert_sel": 3, "pert_val": 4, "index": 5,
             "perm": 6, "noise": 7}
@@ -109,6 +110,12 @@ def lib() -> C.CDLL:
         L.or_perm_value.restype = C.c_uint64
         L.or_stratum_index.argtypes = [C.c_uint64, C.c_uint64, C.c_uint64, C.c_uint32, C.c_uint64]
         L.or_stratum_index.restype = C.c_uint64
+        L.or_special_count.argtypes = [C.c_double, C.c_uint64]
+        L.or_special_count.restype = C.c_uint64
+        L.or_special_index.argtypes = [C.c_uint64, C.c_uint64, C.c_uint64, C.c_uint32, C.c_uint64]
+        L.or_special_index.restype = C.c_uint64
+        L.or_stratum_of.argtypes = [C.c_uint64, C.c_uint64, C.c_uint64]
+        L.or_stratum_of.restype = C.c_uint64
         L.or_map_uniform.argtypes = [C.c_float, C.c_float, u32p, C.c_uint64, f32p]
         L.or_map_box_muller.argtypes = [u32p, C.c_uint64, f32p]
         L.or_map_f32_to_bf16.argtypes = [f32p, C.c_uint64, u16p]
@@ -236,6 +243,18 @@ def stratum_index(N: int, k: int, seed: int, stream: int, s: int) -> int:
     return lib().or_stratum_index(N, k, seed, stream, s)
 
 
+def special_count(rate: float, N: int) -> int:
+    return lib().or_special_count(rate, N)
+
+
+def special_index(N: int, k: int, seed: int, stream: int, s: int) -> int:
+    return lib().or_special_index(N, k, seed, stream, s)
+
+
+def stratum_of(g: int, k: int, N: int) -> int:
+    return lib().or_stratum_of(g, k, N)
+
+
 # ---------------------------------------------------------------------------
 # marshalling of the neutral descriptions
 # ---------------------------------------------------------------------------
@@ -245,7 +264,7 @@ def _perturb(p) -> Perturb:
 
 
 def to_spec(s) -> Spec:
-    mask = 0
+    mask = SPECIAL_EXACT if getattr(s, "special_exact", False) else 0
     for k in s.specials:
         mask |= SPECIALS[k]
     return Spec(DTYPES[s.dtype], DISTS[s.dist], s.n, s.seed, s.stream, mask, s.special_rate,

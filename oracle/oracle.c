@@ -268,13 +268,40 @@ uint64_t or_perm_value(uint64_t N, uint64_t seed, uint32_t stream, uint64_t g) {
 /* Exact-count index selection: [0, N) is cut into k strata                */
 /* [floor(s N / k), floor((s+1) N / k)); stratum s contributes one index     */
 /* drawn uniformly inside it (INDEX purpose, block s).  k distinct indices.  */
-uint64_t or_stratum_index(uint64_t N, uint64_t k, uint64_t seed, uint32_t stream, uint64_t s) {
+static uint64_t stratum_index_purpose(uint64_t N, uint64_t k, uint64_t seed, uint32_t stream, uint32_t purpose,
+                                      uint64_t s) {
   uint64_t start = (uint64_t)(((unsigned __int128)s * N) / k);
   uint64_t end = (uint64_t)(((unsigned __int128)(s + 1) * N) / k);
   uint32_t w[4];
-  or_draw(seed, stream, OR_P_INDEX, s, w);
+  or_draw(seed, stream, purpose, s, w);
   uint64_t x = ((uint64_t)w[0] << 32) | w[1];
   return start + mulhi64(x, end - start);
+}
+
+uint64_t or_stratum_index(uint64_t N, uint64_t k, uint64_t seed, uint32_t stream, uint64_t s) {
+  return stratum_index_purpose(N, k, seed, stream, OR_P_INDEX, s);
+}
+
+/* The stratum holding g: stratum s covers [floor(sN/k), floor((s+1)N/k)),   */
+/* so s is the largest value with floor(sN/k) <= g, i.e. with sN < (g+1)k:    */
+/* s = ceil((g+1)k/N) - 1 = floor(((g+1)k - 1)/N), at most k - 1.             */
+uint64_t or_stratum_of(uint64_t g, uint64_t k, uint64_t N) {
+  unsigned __int128 s = (((unsigned __int128)(g + 1) * k) - 1) / N;
+  return s < k ? (uint64_t)s : k - 1;
+}
+
+/* Reading of "0.01% injected" as an exact count (the paper asks only for     */
+/* broad, special-laden inputs, Sec. 4.2.1): round(rate N) specials, at most  */
+/* N, placed one per stratum like the exact-count perturbations but drawn on  */
+/* the SPECIAL_SEL purpose of the spec's own stream.                          */
+uint64_t or_special_count(double rate, uint64_t N) {
+  if (!(rate > 0.0)) return 0;
+  double k = floor(rate * (double)N + 0.5);
+  return k >= (double)N ? N : (uint64_t)k;
+}
+
+uint64_t or_special_index(uint64_t N, uint64_t k, uint64_t seed, uint32_t stream, uint64_t s) {
+  return stratum_index_purpose(N, k, seed, stream, OR_P_SPECIAL_SEL, s);
 }
 
 static uint64_t rate_threshold(double rate) {
@@ -366,21 +393,35 @@ static uint64_t base_value(const or_spec* s, const uint8_t* arena, uint64_t g) {
 /* special values: element g is special iff its SPECIAL_SEL word is below   */
 /* floor(rate * 2^32); its kind is the j-th set bit of the mask with        */
 /* j = floor(w0 * popcount / 2^32), w0..w3 from SPECIAL_KIND block g.       */
-static uint64_t clean_value(const or_spec* s, const uint8_t* arena, uint64_t g) {
-  uint64_t v0 = base_value(s, arena, g);
+/* Selection: with OR_SP_EXACT, g is special iff it is the index drawn in    */
+/* its own stratum (only that stratum's draw can land on g); otherwise iff   */
+/* its SPECIAL_SEL word is below floor(rate * 2^32).                          */
+static int is_special(const or_spec* s, uint64_t g) {
+  if ((s->special_mask & OR_SP_KINDS) == 0) return 0;
+  if (s->special_mask & OR_SP_EXACT) {
+    uint64_t N = logical_len(s), k = or_special_count(s->special_rate, N);
+    if (k == 0) return 0;
+    return or_special_index(N, k, s->seed, s->stream, or_stratum_of(g, k, N)) == g;
+  }
   uint64_t thr = rate_threshold(s->special_rate);
-  if (s->special_mask == 0 || thr == 0) return v0;
+  if (thr == 0) return 0;
   uint32_t w[4];
   or_draw(s->seed, s->stream, OR_P_SPECIAL_SEL, g >> 2, w);
-  if (!((uint64_t)w[g & 3] < thr)) return v0;
+  return (uint64_t)w[g & 3] < thr;
+}
+
+static uint64_t clean_value(const or_spec* s, const uint8_t* arena, uint64_t g) {
+  uint64_t v0 = base_value(s, arena, g);
+  if (!is_special(s, g)) return v0;
+  uint32_t kinds = s->special_mask & OR_SP_KINDS;
   uint32_t kw[4];
   or_draw(s->seed, s->stream, OR_P_SPECIAL_KIND, g, kw);
   uint32_t nkinds = 0;
-  for (int b = 0; b < 32; ++b) nkinds += (s->special_mask >> b) & 1u;
+  for (int b = 0; b < 32; ++b) nkinds += (kinds >> b) & 1u;
   uint32_t pick = (uint32_t)(((uint64_t)kw[0] * nkinds) >> 32);
   uint32_t kind = 0;
   for (int b = 0, seen = 0; b < 32; ++b) {
-    if ((s->special_mask >> b) & 1u) {
+    if ((kinds >> b) & 1u) {
       if ((uint32_t)seen == pick) { kind = 1u << b; break; }
       ++seen;
     }
@@ -532,8 +573,8 @@ int or_check_spec(const or_spec* s, uint64_t arena_bytes) {
         s->a_offset < s->cand_offset + bytes)
       return -1;
   }
-  uint32_t fmask = OR_SP_NAN | OR_SP_PINF | OR_SP_NINF | OR_SP_DENORM | OR_SP_ZERO | OR_SP_DUP;
-  uint32_t imask = OR_SP_ZERO | OR_SP_IMIN | OR_SP_IMAX | OR_SP_DUP;
+  uint32_t fmask = OR_SP_NAN | OR_SP_PINF | OR_SP_NINF | OR_SP_DENORM | OR_SP_ZERO | OR_SP_DUP | OR_SP_EXACT;
+  uint32_t imask = OR_SP_ZERO | OR_SP_IMIN | OR_SP_IMAX | OR_SP_DUP | OR_SP_EXACT;
   if (s->special_mask & ~(fl ? fmask : imask)) return -1;
   uint32_t ek = s->pelem.kind, ck = s->pcount.kind;
   if (ek != OR_PERT_NONE && ek != OR_PERT_RATE_ADD_PM && ek != OR_PERT_REL_NOISE) return -1;

@@ -45,6 +45,11 @@ enum {
   OR_SP_DENORM = 1u << 3, OR_SP_ZERO = 1u << 4, OR_SP_IMIN = 1u << 5,
   OR_SP_IMAX = 1u << 6, OR_SP_DUP = 1u << 7
 };
+/* selection mode bit of the mask: without it each element is special with
+ * probability `rate` (Bernoulli); with it exactly round(rate * N) elements of
+ * the logical array are, one per stratum (see or_special_index) */
+#define OR_SP_EXACT (1u << 31)
+#define OR_SP_KINDS 0xFFu
 /* candidate perturbations */
 enum {
   OR_PERT_NONE = 0, OR_PERT_RATE_ADD_PM = 1, OR_PERT_REL_NOISE = 2,
@@ -115,6 +120,12 @@ void or_box_muller(uint32_t wa, uint32_t wb, float* z0, float* z1);
 int64_t or_int_range_map32(int64_t lo, uint64_t r, uint32_t w);
 uint64_t or_perm_value(uint64_t N, uint64_t seed, uint32_t stream, uint64_t g);
 uint64_t or_stratum_index(uint64_t N, uint64_t k, uint64_t seed, uint32_t stream, uint64_t s);
+/* exact-count special values: how many (round(rate * N), at most N) and the
+ * index drawn in stratum s of [0, N) cut into k strata (SPECIAL_SEL purpose) */
+uint64_t or_special_count(double rate, uint64_t N);
+uint64_t or_special_index(uint64_t N, uint64_t k, uint64_t seed, uint32_t stream, uint64_t s);
+/* the stratum of [0, N) cut into k strata that holds index g */
+uint64_t or_stratum_of(uint64_t g, uint64_t k, uint64_t N);
 
 /* bulk maps for exhaustive pins */
 void or_map_uniform(float a, float b, const uint32_t* w, uint64_t n, float* out);

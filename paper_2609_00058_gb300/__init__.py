@@ -30,6 +30,7 @@ DTYPE_BYTES = {"f32": 4, "f16": 2, "bf16": 2, "i32": 4, "i64": 8, "u32": 4}
 DISTS = {"uniform": 0, "normal": 1, "int_range": 2, "permutation": 3, "dotlike": 4, "raw_bits": 5,
          "constant": 6, "from_arena": 7}
 SPECIALS = {"nan": 1, "pinf": 2, "ninf": 4, "denorm": 8, "zero": 16, "imin": 32, "imax": 64, "dup": 128}
+SPECIAL_EXACT = 1 << 31
 PERTS = {"none": 0, "rate_add_pm": 1, "rel_noise": 2, "count_set": 3, "count_add": 4, "swap_pairs": 5}
 EQUAL_NAN = 1
 STAGE_RUN, STAGE_SKIPPED = 1, 2
@@ -75,6 +76,7 @@ class GenSpec:
     i1: int = 0
     specials: Tuple[str, ...] = ()
     special_rate: float = 0.0
+    special_exact: bool = False  # exactly round(rate * N) specials, one per stratum
     rows: int = 0
     cols: int = 0
     dot_k: int = 0
@@ -236,7 +238,7 @@ def _perturb(p) -> sv_perturb:
 
 
 def to_c_spec(s) -> syn_spec:
-    mask = 0
+    mask = SPECIAL_EXACT if getattr(s, "special_exact", False) else 0
     for k in s.specials:
         mask |= SPECIALS[k]
     return syn_spec(DTYPES[s.dtype], DISTS[s.dist], s.n, s.seed, s.stream, mask, s.special_rate,

@@ -118,10 +118,11 @@ static int check_spec(const syn_spec& s, uint64_t arena) {
   int rc;
   if (s.ref_offset != SV_NO_OUTPUT && (rc = check_range(s.ref_offset, bytes, arena))) return rc;
   if (s.cand_offset != SV_NO_OUTPUT && (rc = check_range(s.cand_offset, bytes, arena))) return rc;
-  const uint32_t fmask = SV_SP_NAN | SV_SP_PINF | SV_SP_NINF | SV_SP_DENORM | SV_SP_ZERO | SV_SP_DUP;
-  const uint32_t imask = SV_SP_ZERO | SV_SP_IMIN | SV_SP_IMAX | SV_SP_DUP;
+  const uint32_t fmask = SV_SP_NAN | SV_SP_PINF | SV_SP_NINF | SV_SP_DENORM | SV_SP_ZERO | SV_SP_DUP | SV_SP_EXACT;
+  const uint32_t imask = SV_SP_ZERO | SV_SP_IMIN | SV_SP_IMAX | SV_SP_DUP | SV_SP_EXACT;
   if (s.special_mask & ~(fl ? fmask : imask)) return SV_EINVAL;
   if (!valid_rate(s.special_rate)) return SV_EINVAL;
+  if (exact_special_count(s) > SV_MAX_COUNT) return SV_ERANGE;  // strata indices stay below 2^21
   if ((s.dist == SV_UNIFORM || s.dist == SV_NORMAL) && !(std::isfinite(s.p0) && std::isfinite(s.p1)))
     return SV_EINVAL;  // finite parameters keep every drawn value finite
   if (s.dist == SV_UNIFORM && !(s.p1 >= s.p0)) return SV_EINVAL;
@@ -604,6 +605,8 @@ int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena
     for (int k = g.begin; k < g.end; ++k) {
       DevSpec& d = tab[k];
       d.fix_begin = fixes;
+      const uint64_t sp_units = fix_special_units(d.s);  // dot-like exact specials: fixup threads
+      fixes += sp_units;
       const uint64_t units = fix_units(d.s);
       if (units == 0) continue;
       const uint64_t N = d.s.logical_n ? d.s.logical_n : d.s.elem_offset + d.s.n;

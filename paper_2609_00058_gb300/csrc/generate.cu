@@ -83,22 +83,10 @@ __device__ __forceinline__ void store4(uint8_t* base, uint64_t i, const typename
 
 // ---------------------------------------------------------------------------
 // exact-count perturbations: the index of stratum st of [0, N) cut into k
-// strata is floor(st N / k) + mulhi64(x, len), x from INDEX block st; a
-// COUNT edit sets or offsets the candidate value there, SWAP_PAIRS exchanges
-// the candidate values of strata 2j and 2j + 1.
+// strata is drawn on the INDEX purpose of the perturbation's stream
+// (stratum_index); a COUNT edit sets or offsets the candidate value there,
+// SWAP_PAIRS exchanges the candidate values of strata 2j and 2j + 1.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ uint64_t stratum_index(const Ctx& c, uint32_t stream, uint64_t k, uint64_t st) {
-  const uint64_t start = (st * c.N) / k, end = ((st + 1) * c.N) / k;  // st < 2^21, N <= 2^40
-  const uint4 w = draw(c.rk, stream, P_INDEX, st);
-  const uint64_t x = ((uint64_t)w.x << 32) | w.y;
-  return start + __umul64hi(x, end - start);
-}
-
-// the stratum holding logical index g: the largest st with floor(st N / k) <= g
-__device__ __forceinline__ uint64_t stratum_of(uint64_t g, uint64_t k, uint64_t N) {
-  return umin(((g + 1) * k - 1) / N, k - 1);  // (g + 1) k < 2^61
-}
-
 // candidate bits at g after a COUNT_SET / COUNT_ADD edit
 template <int DT, int DIST>
 __device__ uint64_t count_edit_bits(const Ctx& c, const sv_perturb& pc, uint64_t g) {
@@ -129,13 +117,59 @@ __device__ __noinline__ void fused_edits(const Ctx& c, const syn_spec& s, uint64
   const uint64_t m = umin(sl - sf + 1, kMaxFusedEdits);
   if (threadIdx.x >= m) return;
   const uint64_t st = sf + threadIdx.x;
-  const uint64_t g = stratum_index(c, pc.stream, k, st);
+  const uint64_t g = stratum_index(c, pc.stream, P_INDEX, k, st);
   if (g < g0 || g >= g1) return;
-  const uint64_t bits = pc.kind == SV_PERT_SWAP_PAIRS ? value_at<DT, DIST>(c, stratum_index(c, pc.stream, k, st ^ 1), 1)
-                                                      : count_edit_bits<DT, DIST>(c, pc, g);
+  const uint64_t bits = pc.kind == SV_PERT_SWAP_PAIRS
+                            ? value_at<DT, DIST>(c, stratum_index(c, pc.stream, P_INDEX, k, st ^ 1), 1)
+                            : count_edit_bits<DT, DIST>(c, pc, g);
   uint8_t* cand = arena + s.cand_offset;
   if constexpr (elem_bytes(DT) == 2) reinterpret_cast<uint16_t*>(cand)[g - s.elem_offset] = (uint16_t)bits;
   else reinterpret_cast<T*>(cand)[g - s.elem_offset] = (T)bits;
+}
+
+// one element of a spec's output, index i of the output (not the logical index)
+template <int DT>
+__device__ __forceinline__ void put_elem(uint8_t* out, uint64_t i, uint64_t bits) {
+  using T = typename Store<DT>::T;
+  if constexpr (elem_bytes(DT) == 2) reinterpret_cast<uint16_t*>(out)[i] = (uint16_t)bits;
+  else reinterpret_cast<T*>(out)[i] = (T)bits;
+}
+
+// the candidate's final bits at logical index g: the exact-count edit or
+// swap when g is one of their indices, else the value after the element-wise
+// perturbation (what the generator and the edits together leave there)
+template <int DT, int DIST>
+__device__ uint64_t final_cand_bits(const Ctx& c, const syn_spec& s, uint64_t g) {
+  const sv_perturb& pc = s.pcount;
+  if (pc.kind == SV_PERT_COUNT_SET || pc.kind == SV_PERT_COUNT_ADD || pc.kind == SV_PERT_SWAP_PAIRS) {
+    const uint64_t k = fix_strata(s), st = stratum_of(g, k, c.N);
+    if (stratum_index(c, pc.stream, P_INDEX, k, st) == g)
+      return pc.kind == SV_PERT_SWAP_PAIRS ? value_at<DT, DIST>(c, stratum_index(c, pc.stream, P_INDEX, k, st ^ 1), 1)
+                                           : count_edit_bits<DT, DIST>(c, pc, g);
+  }
+  return value_at<DT, DIST>(c, g, 1);
+}
+
+// exact-count special values in the logical range [g0, g1) that this CTA has
+// just generated: thread t takes strata sf + t, sf + t + kThreads, ...; where
+// a stratum's drawn index falls in the range, the clean output gets the
+// special value and the twin its final value (the element-wise perturbation
+// and any exact-count edit applied).  The caller's __syncthreads() orders
+// these stores after the CTA's generating stores; no other CTA writes
+// [g0, g1).  A range meets about k (g1 - g0) / N strata.
+template <int DT, int DIST>
+__device__ __noinline__ void exact_specials_pass(const Ctx& c, const syn_spec& s, uint64_t g0, uint64_t g1,
+                                                 uint8_t* arena) {
+  const uint64_t k = c.sp_k;
+  const uint64_t sf = stratum_of(g0, k, c.N), sl = stratum_of(g1 - 1, k, c.N);
+  uint8_t* ref = s.ref_offset == SV_NO_OUTPUT ? nullptr : arena + s.ref_offset;
+  uint8_t* cand = s.cand_offset == SV_NO_OUTPUT ? nullptr : arena + s.cand_offset;
+  for (uint64_t st = sf + threadIdx.x; st <= sl; st += kThreads) {
+    const uint64_t g = stratum_index(c, c.stream, P_SPECIAL_SEL, k, st);
+    if (g < g0 || g >= g1) continue;
+    if (ref) put_elem<DT>(ref, g - s.elem_offset, value_at<DT, DIST>(c, g, 0));
+    if (cand) put_elem<DT>(cand, g - s.elem_offset, final_cand_bits<DT, DIST>(c, s, g));
+  }
 }
 
 // base values and special values of the quantum g .. g+3
@@ -208,6 +242,25 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
       if (two) store_quantum<DT>(c, cold, ref, cand, eo + ib, ib, vb, 4);
     }
   } else {
+    if constexpr (one_block_dist<DT, DIST>()) {
+      if (!c.sp_thr) {
+        // no per-element special selection (none, or the exact mode): one
+        // VALUE block per quantum, so two quanta per iteration keep two
+        // independent Philox chains in flight
+        for (; q + kThreads < qfull; q += 2ull * kThreads) {
+          const uint64_t ia = q << 2, ib = (q + kThreads) << 2;
+          const uint64_t ba = (eo + ia) >> 2, bb = (eo + ib) >> 2;
+          uint4 wa = make_uint4((uint32_t)ba, (uint32_t)(ba >> 32), c.stream, P_VALUE);
+          uint4 wb = make_uint4((uint32_t)bb, (uint32_t)(bb >> 32), c.stream, P_VALUE);
+          philox2_rk(wa, wb, c.rk);
+          T va[4], vb[4];
+          base4_words<DT, DIST>(c, wa, va);
+          base4_words<DT, DIST>(c, wb, vb);
+          store_quantum<DT>(c, cold, ref, cand, eo + ia, ia, va, 4);
+          store_quantum<DT>(c, cold, ref, cand, eo + ib, ib, vb, 4);
+        }
+      }
+    }
     for (; q < qfull; q += kThreads) {
       T v[4];
       const uint64_t i = q << 2;
@@ -251,6 +304,10 @@ __global__ void __launch_bounds__(kThreads, SV_GEN_MINB) gen_kernel(const __grid
     __syncthreads();
     const uint64_t i0 = (lo - q_base) * 4, i1 = umin((hi - q_base) * 4, cur.s.n);
     gen_run<DT, DIST>(ctx, cur.s, i0, i1, p.arena);
+    if (ctx.sp_k) {  // exact-count special values inside this CTA's range
+      __syncthreads();
+      exact_specials_pass<DT, DIST>(ctx, cur.s, cur.s.elem_offset + i0, cur.s.elem_offset + i1, p.arena);
+    }
     if (cur.fused) {  // uniform: the spec's exact-count edits inside this CTA's range
       __syncthreads();
       fused_edits<DT, DIST>(ctx, cur.s, cur.s.elem_offset + i0, cur.s.elem_offset + i1, p.arena);
@@ -288,6 +345,16 @@ static const void* gen_kernel_for(uint32_t dtype, uint32_t dist) {
 template <int DT, int DIST>
 __device__ void fix_one(const Ctx& c, const syn_spec& s, uint64_t u, uint8_t* arena) {
   using T = typename Store<DT>::T;
+  const uint64_t nsp = fix_special_units(s);
+  if (u < nsp) {  // dot-like values: the exact-count special value of stratum u
+    const uint64_t g = stratum_index(c, c.stream, P_SPECIAL_SEL, c.sp_k, u);
+    if (g < s.elem_offset || g >= s.elem_offset + s.n) return;
+    if (s.ref_offset != SV_NO_OUTPUT) put_elem<DT>(arena + s.ref_offset, g - s.elem_offset, value_at<DT, DIST>(c, g, 0));
+    if (s.cand_offset != SV_NO_OUTPUT)
+      put_elem<DT>(arena + s.cand_offset, g - s.elem_offset, final_cand_bits<DT, DIST>(c, s, g));
+    return;
+  }
+  u -= nsp;
   const sv_perturb& pc = s.pcount;
   uint8_t* cand = arena + s.cand_offset;
   const uint64_t lo = s.elem_offset, hi = s.elem_offset + s.n;
@@ -300,13 +367,14 @@ __device__ void fix_one(const Ctx& c, const syn_spec& s, uint64_t u, uint8_t* ar
   };
   if (pc.kind == SV_PERT_SWAP_PAIRS) {
     const uint64_t k = 2 * pc.count;
-    const uint64_t a = stratum_index(c, pc.stream, k, 2 * u), b = stratum_index(c, pc.stream, k, 2 * u + 1);
+    const uint64_t a = stratum_index(c, pc.stream, P_INDEX, k, 2 * u);
+    const uint64_t b = stratum_index(c, pc.stream, P_INDEX, k, 2 * u + 1);
     const uint64_t va = value_at<DT, DIST>(c, a, 1), vb = value_at<DT, DIST>(c, b, 1);
     put(a, vb);
     put(b, va);
     return;
   }
-  const uint64_t g = stratum_index(c, pc.stream, pc.count, u);
+  const uint64_t g = stratum_index(c, pc.stream, P_INDEX, pc.count, u);
   if (g < lo || g >= hi) return;
   put(g, count_edit_bits<DT, DIST>(c, pc, g));
 }

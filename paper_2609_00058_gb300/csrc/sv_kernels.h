@@ -7,6 +7,7 @@
 #pragma once
 
 #include <cuda_runtime.h>
+#include <math.h>
 #include <stdint.h>
 
 #include "../../include/synverify.h"
@@ -110,6 +111,23 @@ SV_HD inline uint64_t fix_units(const syn_spec& s) {
   if (s.cand_offset == SV_NO_OUTPUT) return 0;
   const uint32_t k = s.pcount.kind;
   return (k == SV_PERT_COUNT_SET || k == SV_PERT_COUNT_ADD || k == SV_PERT_SWAP_PAIRS) ? s.pcount.count : 0;
+}
+
+
+// exact-count special values of a spec: round(rate * N), at most N (the
+// same fp64 steps on the host and the device); 0 in the Bernoulli mode or
+// with no kind in the mask
+SV_HD inline uint64_t exact_special_count(const syn_spec& s) {
+  if (!(s.special_mask & SV_SP_EXACT) || !(s.special_mask & SV_SP_KINDS) || !(s.special_rate > 0.0)) return 0;
+  const uint64_t N = s.logical_n ? s.logical_n : s.elem_offset + s.n;
+  const double k = floor(s.special_rate * (double)N + 0.5);
+  return k >= (double)N ? N : (uint64_t)k;
+}
+
+// fixup threads that write exact-count special values: the dot-like values'
+// (their generator writes none); the streaming generator's CTAs write their own
+SV_HD inline uint64_t fix_special_units(const syn_spec& s) {
+  return s.dist == SV_DOTLIKE ? exact_special_count(s) : 0;
 }
 
 // strata the exact-count edits cut [0, N) into (two per swapped pair)

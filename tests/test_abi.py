@@ -320,3 +320,14 @@ def test_binding_refuses_host_and_strided_tensors_before_any_launch():
     strided = torch.zeros(8192, dtype=torch.uint8)[::2]
     with pytest.raises(ValueError):
         sv.compare(pairs, strided, strided)
+
+
+def test_exact_specials_validation(lib):
+    n = 1 << 22
+    # 2^22 * 0.5 = 2^21 exact specials: beyond SV_MAX_COUNT (2^20) -> SV_ERANGE
+    too_many = sv.SpecTable([W.GenSpec("f32", "uniform", n, ref_offset=0, p0=0, p1=1, specials=("nan",),
+                                       special_rate=0.5, special_exact=True)])
+    assert lib.sv_check_specs(too_many.arr, 1, 4 * n) == -3
+    ok = sv.SpecTable([W.GenSpec("f32", "uniform", n, ref_offset=0, p0=0, p1=1, specials=("nan",),
+                                 special_rate=0.25, special_exact=True)])
+    assert lib.sv_check_specs(ok.arr, 1, 4 * n) == 0

@@ -115,6 +115,15 @@ ALL_SPECS = [
     dict(dtype="f32", dist="constant", p0=2.5),
     dict(dtype="bf16", dist="constant", p0=float("nan")),
     dict(dtype="i64", dist="constant", i0=-7),
+    # exact-count special values: round(rate * N), one per stratum
+    dict(dtype="f32", dist="normal", p0=5.0, p1=10.0, specials=("nan", "pinf", "ninf", "denorm", "zero", "dup"),
+         special_rate=0.01, special_exact=True),
+    dict(dtype="bf16", dist="uniform", p0=-100.0, p1=100.0, specials=("nan", "denorm", "dup"), special_rate=3e-3,
+         special_exact=True),
+    dict(dtype="i64", dist="permutation", specials=("dup", "zero", "imin", "imax"), special_rate=0.01,
+         special_exact=True),
+    dict(dtype="i32", dist="int_range", i0=-100, i1=100, specials=("zero", "imin", "imax"), special_rate=1.0,
+         special_exact=True),  # every element special: every edit lands on a special
 ]
 PERTS = [
     (W.Perturb(), W.Perturb()),
@@ -379,3 +388,69 @@ def test_candidate_pass_from_the_reference_equals_the_fused_twin(dev):
     sv.generate([twin], a)
     h = a.cpu().numpy()
     assert np.array_equal(h[d.cand_offset: d.cand_offset + 2 * n], h[wl.arena_bytes: wl.arena_bytes + 2 * n])
+
+
+# ---------------------------------------------------------------------------
+# exact-count special values (one per stratum; SV_SP_EXACT)
+# ---------------------------------------------------------------------------
+def test_exact_specials_at_a_ladder_stage(dev):
+    """A 2^22 fp32 N(0,1) stage with 1e-3 exact specials (4194 of them, over
+    every CTA of the grid) and one +1e-2 edit: the specials land exactly on
+    the oracle's indices, with its kinds, and nowhere else."""
+    n = 1 << 22
+    spec = W.GenSpec("f32", "normal", n, seed=7, stream=3, ref_offset=0, cand_offset=4 * n, p0=0.0, p1=1.0,
+                     specials=("nan", "pinf", "ninf", "denorm"), special_rate=1e-3, special_exact=True,
+                     pcount=W.Perturb("count_add", stream=103, count=1, value=1e-2))
+    import torch
+    a = torch.zeros(8 * n, dtype=torch.uint8, device=dev)
+    sv.generate([spec], a)
+    h = np.zeros(8 * n, np.uint8)
+    oracle.generate([spec], h, threads=0)
+    g = a.cpu().numpy()
+    check_spec_outputs(g, h, spec)
+    k = oracle.special_count(1e-3, n)
+    idx = [oracle.special_index(n, k, 7, 3, s) for s in range(k)]
+    gv = _view(g, 0, "f32", n)
+    special = ~np.isfinite(gv.view(np.float32)) | ((gv & 0x7F800000) == 0)
+    assert np.nonzero(special)[0].tolist() == idx
+    assert np.array_equal(gv[idx], _view(h, 0, "f32", n)[idx])
+
+
+def test_exact_specials_chunked_and_with_swaps(dev):
+    n = 70_000
+    base = dict(dtype="f32", dist="uniform", seed=3, stream=1, p0=-2.0, p1=3.0, specials=("nan", "dup", "zero"),
+                special_rate=4e-3, special_exact=True,
+                pelem=W.Perturb("rate_add_pm", stream=2, rate=0.01, value=0.5),
+                pcount=W.Perturb("swap_pairs", stream=3, count=9))
+    whole = W.GenSpec(n=n, ref_offset=0, cand_offset=4 * n, **base)
+    cuts = [0, 8192, 8196, 40000, n]
+    chunks = [W.GenSpec(n=c1 - c0, ref_offset=4 * c0, cand_offset=4 * n + 4 * c0, elem_offset=c0, logical_n=n,
+                        **base) for c0, c1 in zip(cuts[:-1], cuts[1:])]
+    import torch
+    a = torch.zeros(8 * n, dtype=torch.uint8, device=dev)
+    b = torch.zeros(8 * n, dtype=torch.uint8, device=dev)
+    sv.generate([whole], a)
+    sv.generate(chunks, b)
+    assert torch.equal(a, b)
+    h = np.zeros(8 * n, np.uint8)
+    oracle.generate([whole], h)
+    assert np.array_equal(a.cpu().numpy(), h)
+
+
+@pytest.mark.parametrize("rate", [0.01, 1.0])
+def test_exact_specials_on_dotlike_values(dev, rate):
+    """Dot-like values take their exact specials from the fixup kernel; at
+    rate 1 every element is special, so every edit lands on one."""
+    rows, cols, k = 65, 132, 33
+    ar = W.Arena()
+    ao, bo = ar.take(4 * rows * k), ar.take(4 * k * cols)
+    ro, co = ar.take(2 * rows * cols), ar.take(2 * rows * cols)
+    fa = W.GenSpec("f32", "uniform", rows * k, seed=1, stream=0, ref_offset=ao, p0=-1, p1=1)
+    fb = W.GenSpec("f32", "uniform", k * cols, seed=1, stream=1, ref_offset=bo, p0=-1, p1=1)
+    d = W.GenSpec("bf16", "dotlike", rows * cols, seed=1, stream=2, ref_offset=ro, cand_offset=co, rows=rows,
+                  cols=cols, dot_k=k, a_offset=ao, b_offset=bo, specials=("nan", "zero", "dup"), special_rate=rate,
+                  special_exact=True, pelem=W.Perturb("rate_add_pm", stream=5, rate=0.05, value=0.25),
+                  pcount=W.Perturb("count_add", stream=6, count=7, value=1.0))
+    g, h = gen_both(dev, [[fa, fb], [d]], ar.size)
+    assert np.array_equal(g, h)
+

@@ -58,6 +58,7 @@ class GenSpec:
     i1: int = 0
     specials: Tuple[str, ...] = ()
     special_rate: float = 0.0
+    special_exact: bool = False  # exactly round(rate * N) specials, one per stratum
     rows: int = 0
     cols: int = 0
     dot_k: int = 0
@@ -166,7 +167,8 @@ LADDER_EXPONENTS = (10, 14, 18, 22, 25, 27)
 def progressive_ladder(exponents: Sequence[int] = LADDER_EXPONENTS, deviate_stage: Optional[int] = 3,
                        special_rate: float = 1e-4) -> Workload:
     """Size-ascending ladder of fp32 N(0,1) stages (seed 7, stream = stage),
-    0.01% injected NaN/+Inf/-Inf/denormal; the candidate equals the reference
+    0.01% injected NaN/+Inf/-Inf/denormal (exactly round(1e-4 N) of them per
+    stage, one per stratum); the candidate equals the reference
     except for one element moved by +1e-2 at stage `deviate_stage` (0-based),
     so validation stops there.  atol = rtol = 1e-5."""
     ar = Arena()
@@ -177,7 +179,7 @@ def progressive_ladder(exponents: Sequence[int] = LADDER_EXPONENTS, deviate_stag
         pc = Perturb("count_add", stream=100 + s, count=1, value=1e-2) if s == deviate_stage else Perturb()
         specs.append(GenSpec("f32", "normal", n, seed=7, stream=s, ref_offset=ref, cand_offset=cand,
                              p0=0.0, p1=1.0, specials=("nan", "pinf", "ninf", "denorm"),
-                             special_rate=special_rate, pcount=pc))
+                             special_rate=special_rate, special_exact=True, pcount=pc))
         pairs.append(Pair("f32", n, cand, ref, atol=1e-5, rtol=1e-5))
     name = "progressive ladder n=2^{%s} fp32 N(0,1)" % ",".join(str(e) for e in exponents)
     return Workload(name, [specs], pairs, ar.size, progressive=True)
