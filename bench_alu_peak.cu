@@ -2,8 +2,9 @@
 // ALU roofline of the dot-like synthesis (K fp32 fused multiply-adds per
 // output, which no memory bound limits).
 //
-// Three plain kernels, none of them the library's code:
+// Four plain kernels, none of them the library's code:
 //   ffma   8 independent fma.rn.f32 chains per thread     -> fp32 FMA / s
+//   ffma2  8 independent fma.rn.f32x2 chains per thread   -> fp32 FMA / s (2 per instruction)
 //   imad   8 independent mad.lo.u32 chains per thread     -> 32-bit IMAD / s
 //   wide   8 independent mad.wide.u32 chains per thread   -> 32x32->64 IMAD / s
 // Grid: 8 CTAs of 256 threads per SM, every thread the same fixed number of
@@ -36,6 +37,35 @@ __global__ void __launch_bounds__(kThreads) ffma_kernel(float* out, float a, flo
   float s = 0.0f;
 #pragma unroll
   for (int j = 0; j < kChains; ++j) s += c[j];
+  out[(size_t)blockIdx.x * kThreads + threadIdx.x] = s;
+  if (threadIdx.x == 0) cycles[blockIdx.x] = clock64() - t0;
+}
+
+// packed pairs: one fma.rn.f32x2 is two fp32 fused multiply-adds
+__global__ void __launch_bounds__(kThreads) ffma2_kernel(float* out, float a, float b, long long* cycles) {
+  const long long t0 = clock64();
+  unsigned long long c[kChains];
+  unsigned long long a2, b2;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(a2) : "f"(a), "f"(a));
+  asm("mov.b64 %0, {%1, %2};" : "=l"(b2) : "f"(b), "f"(b));
+#pragma unroll
+  for (int j = 0; j < kChains; ++j) {
+    const float lo = (float)(threadIdx.x + j), hi = (float)(threadIdx.x + 2 * j);
+    asm("mov.b64 %0, {%1, %2};" : "=l"(c[j]) : "f"(lo), "f"(hi));
+  }
+  for (int i = 0; i < kIters; ++i) {
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u)
+#pragma unroll
+      for (int j = 0; j < kChains; ++j) asm volatile("fma.rn.f32x2 %0, %0, %1, %2;" : "+l"(c[j]) : "l"(a2), "l"(b2));
+  }
+  float s = 0.0f;
+#pragma unroll
+  for (int j = 0; j < kChains; ++j) {
+    float lo, hi;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(c[j]));
+    s += lo + hi;
+  }
   out[(size_t)blockIdx.x * kThreads + threadIdx.x] = s;
   if (threadIdx.x == 0) cycles[blockIdx.x] = clock64() - t0;
 }
@@ -140,9 +170,14 @@ int main() {
   long long* cyc = nullptr;
   CHECK(cudaMalloc(&buf, (size_t)grid * kThreads * sizeof(uint64_t)));
   CHECK(cudaMalloc(&cyc, (size_t)grid * sizeof(long long)));
-  Rate f{}, m{}, w{};
+  Rate f{}, f2{}, m{}, w{};
   if (time_kernel([&] { ffma_kernel<<<grid, kThreads>>>((float*)buf, 0.999999f, 1e-7f, cyc); }, grid, cyc, sms, &f))
     return 1;
+  if (time_kernel([&] { ffma2_kernel<<<grid, kThreads>>>((float*)buf, 0.999999f, 1e-7f, cyc); }, grid, cyc, sms,
+                  &f2))
+    return 1;
+  f2.ops_per_s *= 2;  // two FMAs per packed instruction
+  f2.ops_per_sm_cycle *= 2;
   if (time_kernel([&] { imad_kernel<<<grid, kThreads>>>((uint32_t*)buf, 0x9E3779B9u, 7u, cyc); }, grid, cyc, sms, &m))
     return 1;
   if (time_kernel([&] { wide_kernel<<<grid, kThreads>>>((uint64_t*)buf, 0xD2511F53u, cyc); }, grid, cyc, sms, &w))
@@ -150,9 +185,10 @@ int main() {
   CHECK(cudaFree(buf));
   CHECK(cudaFree(cyc));
   printf("{\"sms\": %d, \"ffma_per_s\": %.6g, \"ffma_per_sm_cycle\": %.4f, \"ffma_mhz\": %.1f, "
+         "\"ffma2_fma_per_s\": %.6g, \"ffma2_fma_per_sm_cycle\": %.4f, "
          "\"imad_per_s\": %.6g, \"imad_per_sm_cycle\": %.4f, \"imad_wide_per_s\": %.6g, "
          "\"imad_wide_per_sm_cycle\": %.4f}\n",
-         sms, f.ops_per_s, f.ops_per_sm_cycle, f.mhz, m.ops_per_s, m.ops_per_sm_cycle, w.ops_per_s,
-         w.ops_per_sm_cycle);
+         sms, f.ops_per_s, f.ops_per_sm_cycle, f.mhz, f2.ops_per_s, f2.ops_per_sm_cycle, m.ops_per_s,
+         m.ops_per_sm_cycle, w.ops_per_s, w.ops_per_sm_cycle);
   return 0;
 }

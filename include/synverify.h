@@ -257,6 +257,32 @@ int sv_check_tiles(const vc_tiles* tiles, size_t cand_bytes, size_t ref_bytes, u
 int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena_bytes, void* d_ws,
                  size_t ws_bytes, sv_stream_t stream);
 
+/* A prepared syn_generate, for callers that synthesize the same spec table
+ * again and again (every candidate of an evolution round is checked on the
+ * same synthesized stages, Sec. 4.2.1/4.2.2): the table is validated,
+ * grouped, scheduled and (beyond SV_INLINE_ENTRIES specs) copied into the
+ * workspace once, so that each syn_generate_planned call only enqueues its
+ * launches.
+ *   sv_generate_plan_create: specs as syn_generate, checked against an arena
+ *     of arena_bytes; d_ws, ws_bytes >= sv_generate_workspace_bytes() of the
+ *     same table (none needed up to SV_INLINE_ENTRIES specs).  Synchronous: it
+ *     returns once the table is in the workspace.  *plan receives a host
+ *     object owned by the caller.
+ *   syn_generate_planned: the bytes syn_generate writes for the plan's specs,
+ *     into an arena of at least the size the plan was checked against (the
+ *     caller keeps that promise), asynchronous on `stream`.  Nothing else may
+ *     use the workspace while the plan lives.  The plan belongs to the device
+ *     that was current at its creation.
+ *   sv_generate_plan_destroy: frees the host object (NULL: nothing).
+ * Errors: as syn_generate (create: also SV_ERANGE when out of host memory);
+ * planned: SV_EINVAL (null plan or arena), SV_EALIGN (arena not on 16
+ * bytes), SV_ECUDA. */
+typedef struct sv_generate_plan sv_generate_plan;
+int sv_generate_plan_create(const syn_spec* specs, int n_specs, size_t arena_bytes, void* d_ws, size_t ws_bytes,
+                            sv_stream_t stream, sv_generate_plan** plan);
+int syn_generate_planned(const sv_generate_plan* plan, void* d_arena, sv_stream_t stream);
+void sv_generate_plan_destroy(sv_generate_plan* plan);
+
 /* verify_compare: functional validation, Eq. 1 (CUDA-Harness Sec. 4.2.1),
  * one vc_result per pair.
  *   pairs/n_pairs   host array of segments.

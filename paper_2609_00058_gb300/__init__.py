@@ -187,6 +187,9 @@ EXPORTS = [
                                          C.POINTER(C.c_void_p)]),
     ("verify_compare_planned", C.c_int, [_VP, _VP, _VP, _VP, _VP]),
     ("sv_compare_plan_destroy", None, [_VP]),
+    ("sv_generate_plan_create", C.c_int, [C.POINTER(syn_spec), C.c_int, _SZ, _VP, _SZ, _VP, C.POINTER(C.c_void_p)]),
+    ("syn_generate_planned", C.c_int, [_VP, _VP, _VP]),
+    ("sv_generate_plan_destroy", None, [_VP]),
     ("sv_check_tiles", C.c_int, [C.POINTER(vc_tiles), _SZ, _SZ, C.POINTER(C.c_uint64)]),
     ("verify_compare_tiles", C.c_int, [C.POINTER(vc_tiles), _VP, _SZ, _VP, _SZ, _VP, _VP]),
     # include/sv_io.h
@@ -332,6 +335,38 @@ def compare(pairs, cand, ref, results=None, workspace=None, stream=None):
                               results.data_ptr(), ws[0], ws[1] if ws[0] else 0, _stream_ptr(stream))
     _ok(rc, "verify_compare")
     return results
+
+
+class GeneratePlan:
+    """sv_generate_plan_create: a syn_generate whose spec table is validated,
+    grouped, scheduled and staged once (in a workspace this object owns), for
+    arenas of at least arena_bytes."""
+
+    def __init__(self, specs, arena_bytes: int, device=None, stream=None):
+        import torch
+        self.tab = specs if isinstance(specs, SpecTable) else SpecTable(specs)
+        self.arena_bytes = arena_bytes
+        dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+        self._ws = _workspace(self.tab.ws_bytes, dev, None)
+        self._h = C.c_void_p()
+        rc = lib().sv_generate_plan_create(self.tab.arr, self.tab.n, arena_bytes, self._ws[0],
+                                           self._ws[1] if self._ws[0] else 0, _stream_ptr(stream), C.byref(self._h))
+        _ok(rc, "sv_generate_plan_create")
+        self.n = self.tab.n
+        self.device = dev
+
+    def __call__(self, arena, stream=None) -> None:
+        """syn_generate_planned into `arena`."""
+        _dense_cuda(arena, "arena")
+        if _nbytes(arena) < self.arena_bytes:
+            raise ValueError("arena smaller than the plan was made for")
+        _ok(lib().syn_generate_planned(self._h, arena.data_ptr(), _stream_ptr(stream)), "syn_generate_planned")
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h is not None and h.value and _lib is not None:
+            _lib.sv_generate_plan_destroy(h)
+            self._h = None
 
 
 class ComparePlan:

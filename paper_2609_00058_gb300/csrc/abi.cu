@@ -443,7 +443,79 @@ static int run_pair_plan(const DevPair* host, const DevPair* dev, int n_pairs, c
   return status_of(launch_combine(host, dev, n_pairs, partials, results, nullptr, 0, st));
 }
 
+// the plan of one syn_generate: the spec table grouped by dtype x
+// distribution (stable), each group's weighted units and launch shape, every
+// spec's first unit, and its exact-count fixup threads -- edits are applied by
+// the generating CTAs where a CTA's slice (at most 4 x chunk elements) meets
+// few strata, else by the fixup kernel.  Returns the fixup threads.
+template <class Tab>
+static uint64_t build_spec_plan(const syn_spec* specs, int n_specs, Tab& tab, std::vector<Group>& groups) {
+  std::vector<int> order;
+  group_by(n_specs, [&](int i) { return specs[i].dtype * 8u + specs[i].dist; }, order, groups);
+  for (Group& g : groups) {
+    for (int k = g.begin; k < g.end; ++k) {
+      const syn_spec& s = specs[order[k]];
+      tab[k].s = s;
+      tab[k].work_begin = g.units;
+      tab[k].fused = 0;
+      tab[k].pad = 0;
+      g.units += gen_units(s);
+      g.tiles += gen_tiles(s);
+    }
+    if (g.units) g.sh = generate_shape(tab[g.begin].s.dtype, tab[g.begin].s.dist, g.units, g.tiles);
+  }
+  uint64_t fixes = 0;
+  for (const Group& g : groups) {
+    for (int k = g.begin; k < g.end; ++k) {
+      DevSpec& d = tab[k];
+      d.fix_begin = fixes;
+      fixes += fix_special_units(d.s);  // dot-like exact specials: fixup threads
+      const uint64_t units = fix_units(d.s);
+      if (units == 0) continue;
+      const uint64_t N = d.s.logical_n ? d.s.logical_n : d.s.elem_offset + d.s.n;
+      if (d.s.dist != SV_DOTLIKE && 4 * g.sh.chunk / N * fix_strata(d.s) +
+                                            (4 * g.sh.chunk % N) * fix_strata(d.s) / N + 2 <= kMaxFusedEdits) {
+        d.fused = 1;
+        continue;
+      }
+      fixes += units;
+    }
+  }
+  return fixes;
+}
+
+// the launches of a generator plan: one per group (one per spec for dot-like
+// values), then the fixup
+static int run_spec_plan(const DevSpec* host, const DevSpec* dev, int n_specs, const std::vector<Group>& groups,
+                         uint64_t fixes, uint8_t* arena, cudaStream_t st) {
+  cudaError_t e = cudaSuccess;
+  for (const Group& g : groups) {
+    const DevSpec& first = host[g.begin];
+    if (first.s.dist == SV_DOTLIKE) {
+      for (int k = g.begin; e == cudaSuccess && k < g.end; ++k) e = launch_dotlike(host[k], arena, st);
+    } else {
+      e = launch_generate_group(first.s.dtype, first.s.dist, host + g.begin, dev ? dev + g.begin : nullptr,
+                                g.end - g.begin, g.units, g.sh, arena, st);
+    }
+    if (e != cudaSuccess) return SV_ECUDA;
+  }
+  return status_of(launch_fixup(host, dev, n_specs, fixes, arena, st));
+}
+
 }  // namespace sv
+
+// a prepared syn_generate (synverify.h): the grouped spec table, kept on the
+// host for the launch parameters and, beyond SV_INLINE_ENTRIES specs, in the
+// caller's workspace for the kernels
+struct sv_generate_plan {
+  int n = 0;
+  size_t arena_bytes = 0;
+  int device = -1;
+  std::vector<sv::DevSpec> tab;
+  std::vector<sv::Group> groups;
+  uint64_t fixes = 0;
+  const sv::DevSpec* dev_tab = nullptr;
+};
 
 // a prepared verify_compare (synverify.h): the grouped table, kept on the host
 // for the launch parameters and, beyond SV_INLINE_ENTRIES pairs, in the
@@ -582,61 +654,58 @@ int syn_generate(const syn_spec* specs, int n_specs, void* d_arena, size_t arena
   const size_t need = spec_table_bytes(n_specs);
   if (!ws_ok(d_ws, ws_bytes, need)) return SV_EWORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  std::vector<int> order;
   std::vector<Group> groups;
-  group_by(n_specs, [&](int i) { return specs[i].dtype * 8u + specs[i].dist; }, order, groups);
   HostTable<DevSpec> tab(n_specs, need != 0);
-  for (Group& g : groups) {
-    for (int k = g.begin; k < g.end; ++k) {
-      const syn_spec& s = specs[order[k]];
-      tab[k].s = s;
-      tab[k].work_begin = g.units;
-      tab[k].fused = 0;
-      tab[k].pad = 0;
-      g.units += gen_units(s);
-      g.tiles += gen_tiles(s);
-    }
-    if (g.units) g.sh = generate_shape(tab[g.begin].s.dtype, tab[g.begin].s.dist, g.units, g.tiles);
-  }
-  // exact-count edits: applied by the generating CTAs where a CTA's slice (at
-  // most 4 x chunk elements) meets few strata, else by the fixup kernel
-  uint64_t fixes = 0;
-  for (const Group& g : groups) {
-    for (int k = g.begin; k < g.end; ++k) {
-      DevSpec& d = tab[k];
-      d.fix_begin = fixes;
-      const uint64_t sp_units = fix_special_units(d.s);  // dot-like exact specials: fixup threads
-      fixes += sp_units;
-      const uint64_t units = fix_units(d.s);
-      if (units == 0) continue;
-      const uint64_t N = d.s.logical_n ? d.s.logical_n : d.s.elem_offset + d.s.n;
-      if (d.s.dist != SV_DOTLIKE && 4 * g.sh.chunk / N * fix_strata(d.s) +
-                                            (4 * g.sh.chunk % N) * fix_strata(d.s) / N + 2 <= kMaxFusedEdits) {
-        d.fused = 1;
-        continue;
-      }
-      fixes += units;
-    }
-  }
+  const uint64_t fixes = build_spec_plan(specs, n_specs, tab, groups);
   const DevSpec* dev = nullptr;
   if (need) {
     if (tab.upload(d_ws, st) != cudaSuccess) return SV_ECUDA;
     dev = static_cast<const DevSpec*>(d_ws);
   }
-  uint8_t* arena = static_cast<uint8_t*>(d_arena);
-  cudaError_t e = cudaSuccess;
-  for (const Group& g : groups) {
-    const DevSpec& first = tab[g.begin];
-    if (first.s.dist == SV_DOTLIKE) {
-      for (int k = g.begin; e == cudaSuccess && k < g.end; ++k) e = launch_dotlike(tab[k], arena, st);
-    } else {
-      e = launch_generate_group(first.s.dtype, first.s.dist, tab.data() + g.begin, dev ? dev + g.begin : nullptr,
-                                g.end - g.begin, g.units, g.sh, arena, st);
-    }
-    if (e != cudaSuccess) return SV_ECUDA;
-  }
-  return status_of(launch_fixup(tab.data(), dev, n_specs, fixes, arena, st));
+  return run_spec_plan(tab.data(), dev, n_specs, groups, fixes, static_cast<uint8_t*>(d_arena), st);
 }
+
+int sv_generate_plan_create(const syn_spec* specs, int n_specs, size_t arena_bytes, void* d_ws, size_t ws_bytes,
+                            sv_stream_t stream, sv_generate_plan** plan) {
+  if (!plan) return SV_EINVAL;
+  *plan = nullptr;
+  if (int rc = check_specs(specs, n_specs, arena_bytes)) return rc;
+  const size_t need = spec_table_bytes(n_specs);
+  if (!ws_ok(d_ws, ws_bytes, need)) return SV_EWORKSPACE;
+  sv_generate_plan* p = new (std::nothrow) sv_generate_plan();
+  if (!p) return SV_ERANGE;
+  p->n = n_specs;
+  p->arena_bytes = arena_bytes;
+  if (cudaGetDevice(&p->device) != cudaSuccess) p->device = -1;
+  if (n_specs > 0) {
+    p->tab.resize((size_t)n_specs);
+    p->fixes = build_spec_plan(specs, n_specs, p->tab, p->groups);
+    if (need) {  // the table goes up once; the plan's launches read it from the workspace
+      cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+      if (cudaMemcpyAsync(d_ws, p->tab.data(), sizeof(DevSpec) * (size_t)n_specs, cudaMemcpyHostToDevice, st) !=
+              cudaSuccess ||
+          cudaStreamSynchronize(st) != cudaSuccess) {
+        cudaGetLastError();
+        delete p;
+        return SV_ECUDA;
+      }
+      p->dev_tab = static_cast<const DevSpec*>(d_ws);
+    }
+  }
+  *plan = p;
+  return SV_OK;
+}
+
+int syn_generate_planned(const sv_generate_plan* plan, void* d_arena, sv_stream_t stream) {
+  if (!plan) return SV_EINVAL;
+  if (plan->n == 0) return SV_OK;
+  if (!d_arena) return SV_EINVAL;
+  if (misaligned(d_arena, 16)) return SV_EALIGN;
+  return run_spec_plan(plan->tab.data(), plan->dev_tab, plan->n, plan->groups, plan->fixes,
+                       static_cast<uint8_t*>(d_arena), reinterpret_cast<cudaStream_t>(stream));
+}
+
+void sv_generate_plan_destroy(sv_generate_plan* plan) { delete plan; }
 
 int verify_compare(const vc_pair* pairs, int n_pairs, const void* d_cand, size_t cand_bytes, const void* d_ref,
                    size_t ref_bytes, vc_result* d_results, void* d_ws, size_t ws_bytes, sv_stream_t stream) {

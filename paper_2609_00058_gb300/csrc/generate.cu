@@ -215,13 +215,21 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
   uint64_t q = q0 + threadIdx.x;
   if constexpr (DIST == SV_FROM_ARENA) {
     // values read from memory, two quanta per iteration: their relative noise
-    // (the usual perturbation of such twins) runs as two interleaved chains
+    // (the usual perturbation of such twins) runs as two interleaved chains.
+    // The next iteration's source vectors are loaded before this iteration's
+    // arithmetic, so their latency overlaps it.
+    T na[4], nb[4];
+    if (q < qfull) base4<DT, DIST>(c, eo + (q << 2), na);
+    if (q + kThreads < qfull) base4<DT, DIST>(c, eo + ((q + kThreads) << 2), nb);
     for (; q < qfull; q += 2ull * kThreads) {
       const uint64_t q2 = q + kThreads, ia = q << 2, ib = q2 << 2;
       const bool two = q2 < qfull;
       T va[4], vb[4];
-      base4<DT, DIST>(c, eo + ia, va);
-      if (two) base4<DT, DIST>(c, eo + ib, vb);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) va[j] = na[j], vb[j] = nb[j];
+      const uint64_t qn = q + 2ull * kThreads;
+      if (qn < qfull) base4<DT, DIST>(c, eo + (qn << 2), na);
+      if (qn + kThreads < qfull) base4<DT, DIST>(c, eo + ((qn + kThreads) << 2), nb);
       if (c.sp_thr) {
         specials4<DT, DIST>(c, cold, eo + ia, va);
         if (two) specials4<DT, DIST>(c, cold, eo + ib, vb);

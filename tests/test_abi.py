@@ -331,3 +331,23 @@ def test_exact_specials_validation(lib):
     ok = sv.SpecTable([W.GenSpec("f32", "uniform", n, ref_offset=0, p0=0, p1=1, specials=("nan",),
                                  special_rate=0.25, special_exact=True)])
     assert lib.sv_check_specs(ok.arr, 1, 4 * n) == 0
+
+
+def test_generate_plan_refusals_before_any_copy(lib):
+    plan = C.c_void_p(123)
+    bad = sv.SpecTable([_spec(ref_offset=8)])  # misaligned output
+    assert lib.sv_generate_plan_create(bad.arr, 1, 4096 * 4, None, 0, None, C.byref(plan)) == -2
+    assert plan.value is None
+    many = sv.SpecTable([_spec(ref_offset=4096 * i) for i in range(9)])  # needs a table in the workspace
+    assert lib.sv_generate_plan_create(many.arr, 9, 4096 * 4 * 9, None, 0, None, C.byref(plan)) == -4
+    good = sv.SpecTable([_spec()])
+    assert lib.sv_generate_plan_create(good.arr, 1, 4096 * 4, None, 0, None, None) == -1
+    assert lib.syn_generate_planned(None, 0x1000, None) == -1
+    # a plan of <= 8 specs needs no workspace and no copy; its calls check the arena
+    assert lib.sv_generate_plan_create(good.arr, 1, 4096 * 4, None, 0, None, C.byref(plan)) == 0
+    try:
+        assert lib.syn_generate_planned(plan, None, None) == -1
+        assert lib.syn_generate_planned(plan, 0x1008, None) == -2
+    finally:
+        lib.sv_generate_plan_destroy(plan)
+    lib.sv_generate_plan_destroy(None)

@@ -454,3 +454,30 @@ def test_exact_specials_on_dotlike_values(dev, rate):
     g, h = gen_both(dev, [[fa, fb], [d]], ar.size)
     assert np.array_equal(g, h)
 
+
+
+@pytest.mark.parametrize("n_specs", [3, 40])
+def test_generate_plan_equals_syn_generate(dev, n_specs):
+    """A plan (table validated, grouped and staged once) writes the bytes of
+    syn_generate, call after call."""
+    import torch
+    kinds = [dict(dtype="f32", dist="normal", p0=5.0, p1=10.0, specials=("nan", "pinf"), special_rate=1e-3,
+                  special_exact=True),
+             dict(dtype="i32", dist="int_range", i0=-5, i1=5),
+             dict(dtype="bf16", dist="uniform", p0=-100.0, p1=100.0, specials=("denorm",), special_rate=0.01),
+             dict(dtype="i64", dist="permutation", pcount=W.Perturb("swap_pairs", stream=4, count=3))]
+    ar = W.Arena()
+    specs = []
+    for i in range(n_specs):
+        kw = kinds[i % len(kinds)]
+        n = [7, 100, 8192, 20001, 65536][i % 5]
+        sz = W.DTYPE_BYTES[kw["dtype"]]
+        specs.append(W.GenSpec(n=n, seed=i, stream=i, ref_offset=ar.take(n * sz), cand_offset=ar.take(n * sz),
+                               **kw))
+    a = torch.zeros(ar.size, dtype=torch.uint8, device=dev)
+    sv.generate(specs, a)
+    plan = sv.GeneratePlan(specs, ar.size, device=dev)
+    for _ in range(2):
+        b = torch.zeros(ar.size, dtype=torch.uint8, device=dev)
+        plan(b)
+        assert torch.equal(a, b)
