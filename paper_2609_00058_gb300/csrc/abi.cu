@@ -59,7 +59,7 @@ unsigned launch_block() {
   return n > 0 ? 0u : (unsigned)kThreads;
 }
 
-uint32_t grid_cap_for(const void* fn, size_t dyn_smem) {
+uint32_t grid_cap_for(const void* fn, size_t dyn_smem, int block) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 152;
   std::lock_guard<std::mutex> lk(g_mu);
@@ -69,7 +69,7 @@ uint32_t grid_cap_for(const void* fn, size_t dyn_smem) {
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 152;
   if (dyn_smem > 0)  // opt in to dynamic shared memory beyond the default 48 KB, once per device
     cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn_smem);
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, dyn_smem) != cudaSuccess || per_sm <= 0)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, block, dyn_smem) != cudaSuccess || per_sm <= 0)
     per_sm = 1;
   const uint32_t cap = (uint32_t)std::min<int>(sms * per_sm, (int)kGridCap);
   g_caps.push_back(CapEntry{dev, fn, cap});

@@ -436,7 +436,15 @@ __global__ void __launch_bounds__(kThreads) fixup_kernel(const __grid_constant__
 #ifndef SV_DOT_MINB
 #define SV_DOT_MINB 2
 #endif
-constexpr int kDotRows = 64, kDotCols = 128, kDotK = 32, kDotStages = SV_DOT_STAGES;
+#ifndef SV_DOT_THREADS
+#define SV_DOT_THREADS 256  // threads per CTA: one warp per 8 rows of the tile
+#endif
+#ifndef SV_DOT_K
+#define SV_DOT_K 32  // k depth of one shared-memory slot (a multiple of 16)
+#endif
+constexpr int kDotThreads = SV_DOT_THREADS;
+constexpr int kDotRows = kDotThreads / 32 * 8, kDotCols = 128, kDotK = SV_DOT_K, kDotStages = SV_DOT_STAGES;
+static_assert(kDotThreads % 32 == 0 && kDotK % 16 == 0, "dot-like tile shape");
 constexpr int kDotSlotFloats = kDotRows * kDotK + kDotK * kDotCols;
 constexpr size_t kDotSmem = (size_t)kDotStages * kDotSlotFloats * sizeof(float);
 
@@ -474,7 +482,7 @@ struct DotCursor {
 
 // A16: the A rows are 16-byte aligned (K % 4 == 0) and move in 16-byte pieces
 template <int DT, bool A16>
-__global__ void __launch_bounds__(kThreads, SV_DOT_MINB) dot_kernel(const __grid_constant__ DotParams p) {
+__global__ void __launch_bounds__(kDotThreads, SV_DOT_MINB) dot_kernel(const __grid_constant__ DotParams p) {
   using T = typename Store<DT>::T;
   extern __shared__ __align__(128) float dsm[];
   __shared__ Ctx cold;
@@ -501,24 +509,24 @@ __global__ void __launch_bounds__(kThreads, SV_DOT_MINB) dot_kernel(const __grid
       float* Bs = As + kDotRows * kDotK;
       if constexpr (A16) {
 #pragma unroll
-        for (int it = 0; it < kDotRows * kDotK / 4 / kThreads; ++it) {
-          const int r = (tid >> 3) + it * (kThreads / 8), q = tid & 7;
+        for (int it = 0; it < kDotRows * kDotK / 4 / kDotThreads; ++it) {
+          const int r = tid / (kDotK / 4) + it * (kDotThreads / (kDotK / 4)), q = tid % (kDotK / 4);
           const uint64_t gr = r0 + r, gk = kc + 4 * q;
           const bool ok = gr < rows && gk < K;  // K % 4 == 0: the whole piece is in range
           cp_async16(As + r * kDotK + 4 * q, ok ? c.A + gr * K + gk : c.A, ok);
         }
       } else {
 #pragma unroll
-        for (int it = 0; it < kDotRows * kDotK / kThreads; ++it) {
-          const int r = (tid >> 5) + it * (kThreads / 32), k = tid & 31;
+        for (int it = 0; it < kDotRows * kDotK / kDotThreads; ++it) {
+          const int r = tid / kDotK + it * (kDotThreads / kDotK), k = tid % kDotK;
           const uint64_t gr = r0 + r, gk = kc + k;
           const bool ok = gr < rows && gk < K;
           cp_async4(As + r * kDotK + k, ok ? c.A + gr * K + gk : c.A, ok);
         }
       }
 #pragma unroll
-      for (int it = 0; it < kDotK * kDotCols / 4 / kThreads; ++it) {
-        const int k = (tid >> 5) + it * (kThreads / 32), q = tid & 31;
+      for (int it = 0; it < kDotK * kDotCols / 4 / kDotThreads; ++it) {
+        const int k = (tid >> 5) + it * (kDotThreads / 32), q = tid & 31;
         const uint64_t gk = kc + k, gc = c0 + 4 * q;
         const bool ok = gk < K && gc < cols;  // cols % 4 == 0
         cp_async16(Bs + k * kDotCols + 4 * q, ok ? c.B + gk * cols + gc : c.B, ok);
@@ -676,9 +684,9 @@ cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_
 template <int DT, bool A16>
 static cudaError_t launch_dot(const DotParams& dp, uint64_t tiles, cudaStream_t st) {
   const void* fn = reinterpret_cast<const void*>(dot_kernel<DT, A16>);
-  const uint32_t cap = grid_cap_for(fn, kDotSmem);
+  const uint32_t cap = grid_cap_for(fn, kDotSmem, kDotThreads);
   const unsigned grid = (unsigned)std::min<uint64_t>(tiles, cap);
-  dot_kernel<DT, A16><<<grid, launch_block(), kDotSmem, st>>>(dp);
+  dot_kernel<DT, A16><<<grid, launch_block() ? kDotThreads : 0u, kDotSmem, st>>>(dp);
   count_launch();
   return cudaGetLastError();
 }

@@ -79,8 +79,9 @@ struct LaunchShape {
 // (align: the chunk is rounded up to a multiple of it, one loop iteration of
 // the kernel, so every slice starts on an iteration boundary)
 LaunchShape shape_for(uint64_t units, uint64_t tiles, uint32_t cap, uint64_t align);
-// SMs x resident CTAs of this kernel (cached per device), at most kGridCap
-uint32_t grid_cap_for(const void* kernel, size_t dyn_smem = 0);
+// SMs x resident CTAs of this kernel at `block` threads per CTA (cached per
+// device), at most kGridCap
+uint32_t grid_cap_for(const void* kernel, size_t dyn_smem = 0, int block = kThreads);
 // one more kernel launched by this library (the sv_kernel_launches counter)
 void count_launch();
 // the block size of every launch: kThreads, or 0 (an invalid configuration,
