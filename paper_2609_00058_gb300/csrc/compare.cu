@@ -170,6 +170,28 @@ __device__ __forceinline__ void fold_vector(Acc& a, float vsum, float vmax, cons
   }
 }
 
+// A vector of matching, finite elements whose only trigger is that some of
+// them (bits of `mask`) may raise the running max |x-y|/|y|: those elements,
+// in order, by the rule of float_elem_full (the other elements need nothing).
+// Returns the updated (max, threshold).
+template <int DT>
+__device__ __noinline__ float2 float_vector_ratio(float maxrel, float relthr, uint4 xv, uint4 yv, uint32_t mask) {
+  constexpr int VE = 16 / elem_bytes(DT);
+  float x[VE], y[VE];
+  unpack_vector<DT>(xv, x);
+  unpack_vector<DT>(yv, y);
+  for (int j = 0; j < VE; ++j) {
+    if (!((mask >> j) & 1u)) continue;
+    const float ay = fabsf(y[j]);
+    const float d = fabsf(__fsub_rn(x[j], y[j]));
+    if (ay != 0.0f && __fmaf_rn(-relthr, ay, d) > 0.0f) {
+      maxrel = fmaxf(maxrel, __fdiv_rn(d, ay));
+      relthr = maxrel;
+    }
+  }
+  return make_float2(maxrel, relthr);
+}
+
 template <int DT>
 __device__ __forceinline__ void float_vector(Acc& a, const Tol& t, const uint4& xv, const uint4& yv, uint64_t idx0) {
   constexpr int VE = 16 / elem_bytes(DT);
@@ -178,19 +200,27 @@ __device__ __forceinline__ void float_vector(Acc& a, const Tol& t, const uint4& 
   unpack_vector<DT>(yv, y);
   float vsum = 0.0f, vmax = 0.0f;
   bool rare = false;
+  uint32_t rel = 0;
 #pragma unroll
   for (int j = 0; j < VE; ++j) {
     const float ay = fabsf(y[j]);
     const float d = fabsf(__fsub_rn(x[j], y[j]));
     const float tol = __fadd_rn(t.atol, __fmul_rn(t.rtol, ay));
     const bool fin = d <= FLT_MAX;
-    rare |= !(d <= tol) | !fin | (__fmaf_rn(-a.relthr, ay, d) > 0.0f);
+    rare |= !(d <= tol) | !fin;
+    rel |= (__fmaf_rn(-a.relthr, ay, d) > 0.0f) ? (1u << j) : 0u;
     dk[j] = fin ? d : 0.0f;
     vmax = fmaxf(vmax, dk[j]);
     vsum = __fmaf_rn(dk[j], dk[j], vsum);
   }
   fold_vector<VE>(a, vsum, vmax, dk);
-  if (rare) a = float_vector_rare<DT>(a, t, xv, yv, idx0);
+  if (rare) {
+    a = float_vector_rare<DT>(a, t, xv, yv, idx0);
+  } else if (rel) {
+    const float2 m = float_vector_ratio<DT>(a.maxrel_f, a.relthr, xv, yv, rel);
+    a.maxrel_f = m.x;
+    a.relthr = m.y;
+  }
 }
 
 // integers: exact equality; statistics only for the (rare) unequal elements,
@@ -329,15 +359,16 @@ __device__ void cmp_run(Acc& a, const vc_pair& pr, const uint8_t* cand, const ui
   if (tail0 < i1 && tid == 0) do_tail<DT>(a, t, xb, yb, tail0, i1);
 }
 
-// warp-wide fold of the accumulators (fixed order); the result is in lane 0
+// fold of the accumulators over aligned groups of `width` lanes (a power of
+// two; 32: the whole warp), in fixed order; each group's result is in its
+// first lane
 template <bool FLOAT>
-__device__ __forceinline__ Partial warp_fold(const Acc& a) {
+__device__ __forceinline__ Partial warp_fold(const Acc& a, int width = 32) {
   uint64_t mism = a.mism, nan_d = a.nan_d, inf_d = a.inf_d, nonfin = a.nonfin, first = a.first;
   double ssq = a.ssq;
   uint64_t maxabs = FLOAT ? (uint64_t)__float_as_uint(a.maxabs_f) : a.maxabs_u;
   double maxrel = FLOAT ? (double)a.maxrel_f : a.maxrel_d;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
+  for (int o = width >> 1; o > 0; o >>= 1) {
     mism += __shfl_down_sync(0xFFFFFFFFu, mism, o);
     nan_d += __shfl_down_sync(0xFFFFFFFFu, nan_d, o);
     inf_d += __shfl_down_sync(0xFFFFFFFFu, inf_d, o);
@@ -558,6 +589,11 @@ struct TileParams {
   const uint8_t* cand;
   const uint8_t* ref;
   vc_result* results;
+  // warp teams only: groups of G full-width tiles side by side (G = 32 / the
+  // tile width in 16-byte vectors; 0: no groups), gpr groups per tile row,
+  // n_groups in all; the other `left` tiles of each tile row one by one
+  uint32_t G;
+  uint64_t gpr, n_groups, left;
 };
 
 // fold b (statistics of other elements) into a; first by minimum
@@ -595,10 +631,66 @@ __device__ __forceinline__ vc_result tile_result(const Partial& q, uint64_t n, b
 // tiles are few and large, or one warp (NT = 32) when there are many, so that
 // the warps of an SM stream their tiles independently (a warp's fold needs no
 // block barrier, and no tile boundary drains the memory pipeline).
-template <int DT, int NT>
-__global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant__ TileParams p) {
+#ifndef SV_TILE_MINB
+#define SV_TILE_MINB 3  // resident CTAs per SM the tile kernel's register budget must allow
+#endif
+#ifndef SV_TILE_U
+#define SV_TILE_U 2  // 16-byte vectors per operand a tile-kernel thread loads per step
+#endif
+#ifndef SV_TILE_GROUP_U
+#define SV_TILE_GROUP_U 4  // rows a tile-group lane loads per step (one 16-byte vector per operand each)
+#endif
+// G side-by-side tiles of one tile row for one warp: lane l owns vector
+// column l of the group (tile l / (32 / G)) and walks down the rows, so every
+// row of the group is one 512-byte run per operand, and the address and the
+// element index advance by one add per row.  The running max |x-y|/|y| is
+// shared within a tile's lanes only (its threshold must not exceed that
+// tile's own maximum).
+template <int DT>
+__device__ __forceinline__ void tile_group(const TileParams& p, uint64_t item, int lane, const Tol& tol) {
   constexpr uint32_t sz = elem_bytes(DT), VE = 16 / sz;
-  constexpr int U = 4;                                // vectors per thread per step
+  constexpr int U = SV_TILE_GROUP_U;
+  const vc_tiles& t = p.t;
+  const int vr = 32 / (int)p.G;  // lanes per tile
+  const uint64_t ti = item / p.gpr, gj = item - ti * p.gpr;
+  const uint64_t r0 = ti * t.tile_rows, col = gj * p.G * t.tile_cols + (uint64_t)lane * VE;
+  const uint32_t h = (uint32_t)(umin(r0 + t.tile_rows, t.rows) - r0);
+  const uint64_t xpb = t.cand_pitch * sz, ypb = t.ref_pitch * sz;
+  const uint8_t* xp = p.cand + t.cand_offset + (r0 * t.cand_pitch + col) * sz;
+  const uint8_t* yp = p.ref + t.ref_offset + (r0 * t.ref_pitch + col) * sz;
+  uint64_t idx = r0 * t.cols + col;
+  Acc a;
+  acc_reset(a);
+  for (uint32_t r = 0; r < h; r += U) {  // h is the same for every lane
+    uint4 x[U], y[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (r + u < h) {
+        x[u] = ldg_stream(reinterpret_cast<const uint4*>(xp + u * xpb));
+        y[u] = ldg_stream(reinterpret_cast<const uint4*>(yp + u * ypb));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (r + u < h) do_vector<DT>(a, tol, x[u], y[u], idx + (uint64_t)u * t.cols);
+    xp += U * xpb;
+    yp += U * ypb;
+    idx += U * t.cols;
+    if constexpr (is_float(DT)) {
+      float m = a.maxrel_f;
+      for (int o = vr >> 1; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+      a.relthr = m;
+    }
+  }
+  const Partial f = warp_fold<is_float(DT)>(a, vr);
+  if (lane % vr == 0)
+    p.results[ti * p.ntc + gj * p.G + (uint64_t)(lane / vr)] = tile_result(f, (uint64_t)h * t.tile_cols, is_float(DT));
+}
+
+template <int DT, int NT>
+__global__ void __launch_bounds__(kThreads, SV_TILE_MINB) tile_kernel(const __grid_constant__ TileParams p) {
+  constexpr uint32_t sz = elem_bytes(DT), VE = 16 / sz;
+  constexpr int U = SV_TILE_U;                        // vectors per thread per step
   constexpr uint32_t kStep = (uint32_t)U * NT;
   constexpr int kTeams = kThreads / NT;               // teams per CTA
   __shared__ Partial tile_sum;
@@ -611,7 +703,14 @@ __global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant
   const uint8_t* yb = p.ref + t.ref_offset;
   // every team runs the same number of rounds (a CTA's barrier needs all its threads)
   const uint64_t rounds = NT == kThreads ? (p.n_tiles + teams - 1) / teams : 0;
-  for (uint64_t k = 0, tile = team; NT == kThreads ? k < rounds : tile < p.n_tiles; ++k, tile += teams) {
+  // warp teams take the tiles outside the groups (all tiles when there are none)
+  const uint64_t items = NT == kThreads ? p.n_tiles : p.n_tiles - p.n_groups * p.G;
+  for (uint64_t k = 0, item = team; NT == kThreads ? k < rounds : item < items; ++k, item += teams) {
+    uint64_t tile = item;
+    if constexpr (NT != kThreads) {
+      const uint64_t tr = item / p.left;
+      tile = tr * p.ntc + p.gpr * p.G + (item - tr * p.left);
+    }
     const bool live = tile < p.n_tiles;
     const uint64_t ti = live ? tile / p.ntc : 0, tj = live ? tile - ti * p.ntc : 0;
     const uint64_t r0 = ti * t.tile_rows, c0 = tj * t.tile_cols;
@@ -687,6 +786,40 @@ __global__ void __launch_bounds__(kThreads, 2) tile_kernel(const __grid_constant
   }
 }
 
+// the groups of side-by-side tiles, one group per warp at a time (a kernel of
+// its own: few registers, so 3 CTAs per SM keep 4 rows of loads in flight)
+template <int DT>
+__global__ void __launch_bounds__(kThreads, 3) tile_group_kernel(const __grid_constant__ TileParams p) {
+  const vc_tiles& t = p.t;
+  const Tol tol{__double2float_rn(t.atol), __double2float_rn(t.rtol), (t.flags & SV_EQUAL_NAN) != 0};
+  const int lane = (int)(threadIdx.x & 31);
+  const uint64_t warps = (uint64_t)gridDim.x * (kThreads / 32);
+  for (uint64_t item = (uint64_t)blockIdx.x * (kThreads / 32) + threadIdx.x / 32; item < p.n_groups; item += warps)
+    tile_group<DT>(p, item, lane, tol);
+}
+
+static const void* tile_group_kernel_for(uint32_t dtype) {
+  switch (dtype) {
+    case SV_F32: return reinterpret_cast<const void*>(&tile_group_kernel<SV_F32>);
+    case SV_F16: return reinterpret_cast<const void*>(&tile_group_kernel<SV_F16>);
+    case SV_BF16: return reinterpret_cast<const void*>(&tile_group_kernel<SV_BF16>);
+    case SV_I32: return reinterpret_cast<const void*>(&tile_group_kernel<SV_I32>);
+    case SV_I64: return reinterpret_cast<const void*>(&tile_group_kernel<SV_I64>);
+    default: return reinterpret_cast<const void*>(&tile_group_kernel<SV_U32>);
+  }
+}
+
+static void launch_tile_groups(const TileParams& tp, uint32_t grid, cudaStream_t st) {
+  switch (tp.t.dtype) {
+    case SV_F32: tile_group_kernel<SV_F32><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_F16: tile_group_kernel<SV_F16><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_BF16: tile_group_kernel<SV_BF16><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_I32: tile_group_kernel<SV_I32><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_I64: tile_group_kernel<SV_I64><<<grid, launch_block(), 0, st>>>(tp); break;
+    default: tile_group_kernel<SV_U32><<<grid, launch_block(), 0, st>>>(tp); break;
+  }
+}
+
 template <int NT>
 static const void* tile_kernel_for(uint32_t dtype) {
   switch (dtype) {
@@ -721,12 +854,32 @@ cudaError_t launch_compare_tiles(const vc_tiles& t, uint64_t ntc, uint64_t n_til
   tp.cand = cand;
   tp.ref = ref;
   tp.results = results;
+  tp.G = 0;
+  tp.gpr = 0;
+  tp.n_groups = 0;
+  tp.left = ntc;
   // one warp per tile once there are enough tiles for every resident warp to
   // hold a few; otherwise the whole CTA shares each tile
   const uint32_t cap_w = grid_cap_for(tile_kernel_for<32>(t.dtype));
   const bool warps = n_tiles >= 4ull * cap_w * (kThreads / 32);
   if (warps) {
-    const uint64_t want = (n_tiles + kThreads / 32 - 1) / (kThreads / 32);
+    // tiles narrower than the output whose width in 16-byte vectors divides
+    // 32 go to the warps in groups of 32 / width side by side
+    const uint64_t vr = t.tile_cols * elem_bytes((int)t.dtype) / 16;  // whole vectors (validated)
+    if (t.tile_cols < t.cols && vr >= 1 && vr <= 32 && 32 % vr == 0) {
+      tp.G = (uint32_t)(32 / vr);
+      tp.gpr = (t.cols / t.tile_cols) / tp.G;
+      tp.left = ntc - tp.gpr * tp.G;
+      tp.n_groups = (n_tiles / ntc) * tp.gpr;
+    }
+    if (tp.n_groups) {  // the groups, then the other tiles one warp each
+      const uint64_t want = (tp.n_groups + kThreads / 32 - 1) / (kThreads / 32);
+      launch_tile_groups(tp, (uint32_t)umin(want, grid_cap_for(tile_group_kernel_for(t.dtype))), st);
+      count_launch();
+    }
+    const uint64_t rest = n_tiles - tp.n_groups * tp.G;
+    if (rest == 0) return cudaGetLastError();
+    const uint64_t want = (rest + kThreads / 32 - 1) / (kThreads / 32);
     launch_tiles<32>(tp, (uint32_t)umin(want, cap_w), st);
   } else {
     launch_tiles<kThreads>(tp, (uint32_t)umin(n_tiles, grid_cap_for(tile_kernel_for<kThreads>(t.dtype))), st);

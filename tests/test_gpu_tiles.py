@@ -68,6 +68,11 @@ CASES = [  # rows, cols, cand pitch, ref pitch, tile rows, tile cols
     (300, 513, 520, 520, 128, 128),
     (10000, 64, 64, 72, 1, 64),      # enough tiles for one warp per tile
     (12000, 37, 40, 48, 1, 37),      # one warp per tile, a ragged end in every row
+    # enough tiles for warp teams, tiles narrower than the output: groups of
+    # side-by-side tiles (their width in vectors divides 32) plus the ragged
+    # last tile column one by one; 7 and 5 rows per tile, padded pitches
+    (16000, 520, 528, 536, 7, 64),
+    (20000, 100, 104, 112, 5, 32),   # (16-bit types: no whole group fits in a row)
 ]
 
 
