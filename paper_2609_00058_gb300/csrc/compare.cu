@@ -171,17 +171,16 @@ __device__ __forceinline__ void fold_vector(Acc& a, float vsum, float vmax, cons
 }
 
 // A vector of matching, finite elements whose only trigger is that some of
-// them (bits of `mask`) may raise the running max |x-y|/|y|: those elements,
-// in order, by the rule of float_elem_full (the other elements need nothing).
-// Returns the updated (max, threshold).
+// them may raise the running max |x-y|/|y|: the max part of float_elem_full
+// over its elements in order (the verdict and the other statistics need
+// nothing more).  Returns the updated (max, threshold).
 template <int DT>
-__device__ __noinline__ float2 float_vector_ratio(float maxrel, float relthr, uint4 xv, uint4 yv, uint32_t mask) {
+__device__ __noinline__ float2 float_vector_ratio(float maxrel, float relthr, uint4 xv, uint4 yv) {
   constexpr int VE = 16 / elem_bytes(DT);
   float x[VE], y[VE];
   unpack_vector<DT>(xv, x);
   unpack_vector<DT>(yv, y);
   for (int j = 0; j < VE; ++j) {
-    if (!((mask >> j) & 1u)) continue;
     const float ay = fabsf(y[j]);
     const float d = fabsf(__fsub_rn(x[j], y[j]));
     if (ay != 0.0f && __fmaf_rn(-relthr, ay, d) > 0.0f) {
@@ -199,8 +198,7 @@ __device__ __forceinline__ void float_vector(Acc& a, const Tol& t, const uint4& 
   unpack_vector<DT>(xv, x);
   unpack_vector<DT>(yv, y);
   float vsum = 0.0f, vmax = 0.0f;
-  bool rare = false;
-  uint32_t rel = 0;
+  bool rare = false, rel = false;
 #pragma unroll
   for (int j = 0; j < VE; ++j) {
     const float ay = fabsf(y[j]);
@@ -208,7 +206,7 @@ __device__ __forceinline__ void float_vector(Acc& a, const Tol& t, const uint4& 
     const float tol = __fadd_rn(t.atol, __fmul_rn(t.rtol, ay));
     const bool fin = d <= FLT_MAX;
     rare |= !(d <= tol) | !fin;
-    rel |= (__fmaf_rn(-a.relthr, ay, d) > 0.0f) ? (1u << j) : 0u;
+    rel |= __fmaf_rn(-a.relthr, ay, d) > 0.0f;
     dk[j] = fin ? d : 0.0f;
     vmax = fmaxf(vmax, dk[j]);
     vsum = __fmaf_rn(dk[j], dk[j], vsum);
@@ -217,7 +215,7 @@ __device__ __forceinline__ void float_vector(Acc& a, const Tol& t, const uint4& 
   if (rare) {
     a = float_vector_rare<DT>(a, t, xv, yv, idx0);
   } else if (rel) {
-    const float2 m = float_vector_ratio<DT>(a.maxrel_f, a.relthr, xv, yv, rel);
+    const float2 m = float_vector_ratio<DT>(a.maxrel_f, a.relthr, xv, yv);
     a.maxrel_f = m.x;
     a.relthr = m.y;
   }

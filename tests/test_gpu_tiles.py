@@ -181,8 +181,10 @@ def test_medium_output_per_tile(dev):
     sampled tile rows are recomputed by the oracle from the same bytes."""
     import torch
     side = 8192
-    ref = torch.randn(side * side, dtype=torch.float32, device=dev) * 10 + 5
-    cand = ref * (1 + torch.randn_like(ref) * 2 ** -9)
+    g = torch.Generator(device=dev)
+    g.manual_seed(8192)
+    ref = torch.randn(side * side, dtype=torch.float32, device=dev, generator=g) * 10 + 5
+    cand = ref * (1 + torch.randn(side * side, dtype=torch.float32, device=dev, generator=g) * 2 ** -9)
     ref16, cand16 = ref.to(torch.bfloat16), cand.to(torch.bfloat16)
     cand16[123456] = float("nan")
     cand16[side * 4000 + 77] += 3.0
@@ -199,4 +201,6 @@ def test_medium_output_per_tile(dev):
             if w["first_mismatch"] >= 0:
                 w["first_mismatch"] += 64 * ti * side
         assert_results_match(got[128 * ti: 128 * ti + 128], want, "tile row %d" % ti)
-    assert sum(g["mismatches"] for g in got) >= 2 and got[62 * 128 + 1]["first_mismatch"] == side * 4000 + 77
+    # the planted +3 is a mismatch of its tile (a natural one may come first)
+    assert sum(r["mismatches"] for r in got) >= 2
+    assert 0 <= got[62 * 128 + 1]["first_mismatch"] <= side * 4000 + 77
