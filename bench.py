@@ -52,19 +52,26 @@ import workloads as W  # noqa: E402
 METRIC = "verified GB/s and synthesized GB/s on 1 GB300, as % of HBM peak"
 L2_BYTES = 129 * 1000 * 1000  # GB300 L2 (bytes, nominal 129 MB)
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-# DRAM bytes per step of each workload's generator and compare kernels from
-# one single-pass ncu launch list (dram__bytes_read.sum + dram__bytes_write.sum
-# summed over the step's launches of that role), keyed by (workload, role,
+# DRAM bytes per step of each workload's generator and compare kernels
+# (dram__bytes_read.sum + dram__bytes_write.sum), keyed by (workload, role,
 # hash of the sources of that role's kernels): a figure taken on other
 # sources is not reported (null)
 NCU_TRAFFIC = {
-    # gen_kernel<f32, normal>, median of the 7 launches of one launch list of
-    # the ladder step: 122,880 B read + 1,312,933,120 B written; the one
-    # exact-count edit is applied by the generating CTA (no fixup launch)
-    ("ladder", "generate", "c7ab7035e73bbe0a"): 1313085696,
-    # gen_kernel<i64, permutation>, median of 7 launches of the permutation
-    # step: 2,013,440 B read + 4,231,760,384 B written; the 34 swap edits fused
-    ("perm_i64", "generate", "c7ab7035e73bbe0a"): 4233829888,
+    # one single-pass launch list per workload (python bench.py --workload W
+    # --only-headline --steps 2 --warmup 1 --no-cpu-baseline): the step's own
+    # launches of each role, summed over its 7 steps and divided by 7
+    ("perm_i64", "generate", "502ee1030ec0bc92"): 4234047415,  # gen_kernel<i64, permutation>, edits fused
+    ("perm_i64", "verify", "cd518aad9c0beae3"): 4295421221,    # cmp_kernel<i64> + combine_kernel
+    ("ladder", "generate", "502ee1030ec0bc92"): 1316616411,    # gen_kernel<f32, normal>, one launch
+    ("ladder", "verify", "cd518aad9c0beae3"): 36020955,        # 3 stage groups: cmp_kernel + combine_stages_kernel
+    ("dotlike_bf16", "generate", "502ee1030ec0bc92"): 4417183122,  # factors gen_kernel + dot_kernel<bf16>
+    ("dotlike_bf16", "verify", "cd518aad9c0beae3"): 4298288640,    # cmp_kernel<bf16> + combine_kernel
+    # the two small workloads' outputs stay in L2 through the step (DRAM
+    # counts only what the caches write back meanwhile)
+    ("segmented", "generate", "502ee1030ec0bc92"): 5687296,
+    ("segmented", "verify", "cd518aad9c0beae3"): 146431890,
+    ("fp32_pair", "generate", "502ee1030ec0bc92"): 76910,
+    ("fp32_pair", "verify", "cd518aad9c0beae3"): 8450158,
 }
 ROLE_SOURCES = {"generate": ("generate.cu", "sv_device.cuh", "sv_kernels.h"),
                 "verify": ("compare.cu", "sv_device.cuh", "sv_kernels.h")}
@@ -306,7 +313,17 @@ def io_reference_arm(args):
 # ---------------------------------------------------------------------------
 # the GPU arm
 # ---------------------------------------------------------------------------
+SMALL = {  # the same kernels on cases of a few GB at most (for ncu captures): --small
+    "dotlike_bf16": lambda: W.dotlike_bf16_pair(rows=8192),
+    "perm_i64": lambda: W.int64_permutation_pair(1 << 26),
+    "ladder": lambda: W.progressive_ladder(W.LADDER_EXPONENTS[:-1]),
+}
+_small = False
+
+
 def full_workload(name):
+    if _small and name in SMALL:
+        return SMALL[name]()
     return W.FULL_SIZE[name]()
 
 
@@ -455,15 +472,14 @@ def measure_workload(name, args, dev, world, steps, warmup, alu):
         # the output compared per 128 x 128 tile (shaped outputs): the same
         # bytes as the verify step, 65536 verdicts instead of one
         pr = wl.pairs[0]
-        side = int(round(pr.n ** 0.5))
-        tt = sv.Tiles(pr.dtype, side, side, pr.cand_offset, pr.ref_offset, tile_rows=128, tile_cols=128,
+        tt = sv.Tiles(pr.dtype, d.rows, d.cols, pr.cand_offset, pr.ref_offset, tile_rows=128, tile_cols=128,
                       atol=pr.atol, rtol=pr.rtol)
         n_t = sv.tile_count(tt, wl.arena_bytes, wl.arena_bytes)
         tres = torch.empty(n_t * sv.RESULT_BYTES, dtype=torch.uint8, device=dev)
         tp_ms = timed_events(stream, lambda: sv.compare_tiles(tt, arena, arena, results=tres), reps)
         tp_bytes = 2 * pr.n * W.DTYPE_BYTES[pr.dtype]
         extra["tile_verify"] = {"what": "verify_compare_tiles, %d x %d output in 128 x 128 tiles (%d verdicts)"
-                                        % (side, side, n_t), "ms": tp_ms, "bytes": tp_bytes,
+                                        % (d.rows, d.cols, n_t), "ms": tp_ms, "bytes": tp_bytes,
                                 "gbs": tp_bytes / (tp_ms * 1e-3) / 1e9,
                                 "frac_of_hbm": tp_bytes / (tp_ms * 1e-3) / 1e9 / hbm}
         if alu:
@@ -822,7 +838,11 @@ def main():
     ap.add_argument("--only-headline", action="store_true", help="measure the --workload alone")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--oracle-threads", type=int, default=0, help="oracle threads (0: every host core)")
+    ap.add_argument("--small", action="store_true",
+                    help="smaller cases of the large workloads (profiling; not the configured sizes)")
     args = ap.parse_args()
+    global _small
+    _small = args.small
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if world > 1:
