@@ -80,6 +80,9 @@ __device__ __forceinline__ void store4(uint8_t* base, uint64_t i, const typename
 #ifndef SV_GEN_MINB
 #define SV_GEN_MINB 2  // resident CTAs per SM the register budget must allow
 #endif
+#ifndef SV_GEN_PIPELINE
+#define SV_GEN_PIPELINE 1  // draw the next iteration's VALUE blocks before this iteration's maps (0: after)
+#endif
 
 // ---------------------------------------------------------------------------
 // exact-count perturbations: the index of stratum st of [0, N) cut into k
@@ -255,6 +258,30 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
         // no per-element special selection (none, or the exact mode): one
         // VALUE block per quantum, so two quanta per iteration keep two
         // independent Philox chains in flight
+#if SV_GEN_PIPELINE
+        // and the next iteration's blocks are drawn before this iteration's
+        // value maps, so the multiply-bound Philox rounds and the
+        // issue-bound maps interleave (the last iteration's look-ahead draw
+        // is for counters past the range: computed, never stored)
+        const uint64_t b0 = (eo >> 2) + q;
+        uint4 wa = make_uint4((uint32_t)b0, (uint32_t)(b0 >> 32), c.stream, P_VALUE);
+        uint4 wb = make_uint4((uint32_t)(b0 + kThreads), (uint32_t)((b0 + kThreads) >> 32), c.stream, P_VALUE);
+        philox2_rk(wa, wb, c.rk);
+        for (; q + kThreads < qfull; q += 2ull * kThreads) {
+          const uint64_t ia = q << 2, ib = (q + kThreads) << 2;
+          const uint64_t bn = (eo >> 2) + q + 2ull * kThreads;
+          uint4 na = make_uint4((uint32_t)bn, (uint32_t)(bn >> 32), c.stream, P_VALUE);
+          uint4 nb = make_uint4((uint32_t)(bn + kThreads), (uint32_t)((bn + kThreads) >> 32), c.stream, P_VALUE);
+          philox2_rk(na, nb, c.rk);
+          T va[4], vb[4];
+          base4_words<DT, DIST>(c, wa, va);
+          base4_words<DT, DIST>(c, wb, vb);
+          store_quantum<DT>(c, cold, ref, cand, eo + ia, ia, va, 4);
+          store_quantum<DT>(c, cold, ref, cand, eo + ib, ib, vb, 4);
+          wa = na;
+          wb = nb;
+        }
+#else
         for (; q + kThreads < qfull; q += 2ull * kThreads) {
           const uint64_t ia = q << 2, ib = (q + kThreads) << 2;
           const uint64_t ba = (eo + ia) >> 2, bb = (eo + ib) >> 2;
@@ -267,6 +294,7 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
           store_quantum<DT>(c, cold, ref, cand, eo + ia, ia, va, 4);
           store_quantum<DT>(c, cold, ref, cand, eo + ib, ib, vb, 4);
         }
+#endif
       }
     }
     for (; q < qfull; q += kThreads) {
