@@ -411,7 +411,6 @@ __device__ void flush(Acc& a, Partial* out) {
 // one instantiation per dtype; the host groups the pairs by dtype
 template <int DT>
 __global__ void __launch_bounds__(kThreads, 3) cmp_kernel(const __grid_constant__ CmpParams p) {
-  __shared__ DevPair cur;
   if (p.flag && *p.flag >= 0) return;  // an earlier stage failed
   __shared__ uint64_t staged[kStagedStarts];
   const uint64_t u0 = (uint64_t)blockIdx.x * p.chunk;
@@ -422,21 +421,20 @@ __global__ void __launch_bounds__(kThreads, 3) cmp_kernel(const __grid_constant_
   acc_reset(a);
   constexpr uint64_t VE = 16 / elem_bytes(DT);
   for (int e = lo; e < p.n; ++e) {
-    __syncthreads();
-    if (threadIdx.x == 0) cur = *pentry(p, e);
-    __syncthreads();
-    const uint64_t wb = cur.work_begin;
+    // every thread reads the segment from the table (no staging, no barrier)
+    const DevPair* te = pentry(p, e);
+    const uint64_t wb = te->work_begin;
     if (wb >= u1) break;
-    const uint64_t we = wb + cmp_units(cur.p);
+    const vc_pair pr = te->p;
+    const uint64_t we = wb + cmp_units(pr);
     if (we <= u0) continue;
     // this CTA overlaps the segment's units: it writes a partial for it (the
     // combine reads one from every overlapping CTA), covering the segment's
     // vectors that fall in [u0, u1) -- units [wb + overhead, we)
-    const vc_pair pr = cur.p;
     const uint64_t v_base = wb + kCmpEntryUnits;
     const uint64_t vlo = umax(u0, v_base), vhi = umin(u1, we);
     if (vhi > vlo) cmp_run<DT>(a, pr, p.cand, p.ref, (vlo - v_base) * VE, umin((vhi - v_base) * VE, pr.n));
-    flush<is_float(DT)>(a, p.partials + cur.slot0 + blockIdx.x);
+    flush<is_float(DT)>(a, p.partials + te->slot0 + blockIdx.x);
   }
 }
 

@@ -320,34 +320,42 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
 // that a launch only sees its own kind
 template <int DT, int DIST>
 __global__ void __launch_bounds__(kThreads, SV_GEN_MINB) gen_kernel(const __grid_constant__ GenParams p) {
-  __shared__ DevSpec cur;
-  __shared__ Ctx ctx;
+  // two slots for the entry in use and its context: an entry is staged into
+  // the slot its predecessor did not use, so one barrier per entry suffices
+  // (a slot's previous user is two entries back, which every thread finished
+  // before passing the last entry's barrier)
+  __shared__ DevSpec cur[2];
+  __shared__ Ctx ctx[2];
   __shared__ uint64_t staged[kStagedStarts];
   const uint64_t u0 = (uint64_t)blockIdx.x * p.chunk;
   const uint64_t u1 = umin(u0 + p.chunk, p.total);
   if (u0 >= u1) return;
+  int slot = 0;
   for (int e = find_start(entry(p, 0), p.n, u0, staged); e < p.n; ++e) {
-    __syncthreads();  // previous entry no longer in use
-    stage_entry(entry(p, e), &cur);
-    __syncthreads();
-    const uint64_t wb = cur.work_begin;
+    // the entry's place in the units, read from the table by every thread
+    const DevSpec* te = entry(p, e);
+    const uint64_t wb = te->work_begin;
     if (wb >= u1) break;
     // this entry's quanta occupy units [wb + overhead, wb + gen_units)
     const uint64_t q_base = wb + kGenEntryUnits;
-    const uint64_t lo = umax(u0, q_base), hi = umin(u1, wb + gen_units(cur.s));
+    const uint64_t lo = umax(u0, q_base), hi = umin(u1, wb + gen_units(te->s));
     if (hi <= lo) continue;
-    if (threadIdx.x == 0) ctx = make_ctx(cur.s, p.arena);
+    stage_entry(te, &cur[slot]);
+    if (threadIdx.x == 0) ctx[slot] = make_ctx(te->s, p.arena);
     __syncthreads();
-    const uint64_t i0 = (lo - q_base) * 4, i1 = umin((hi - q_base) * 4, cur.s.n);
-    gen_run<DT, DIST>(ctx, cur.s, i0, i1, p.arena);
-    if (ctx.sp_k) {  // exact-count special values inside this CTA's range
+    const DevSpec& d = cur[slot];
+    const Ctx& cx = ctx[slot];
+    const uint64_t i0 = (lo - q_base) * 4, i1 = umin((hi - q_base) * 4, d.s.n);
+    gen_run<DT, DIST>(cx, d.s, i0, i1, p.arena);
+    if (cx.sp_k) {  // exact-count special values inside this CTA's range
       __syncthreads();
-      exact_specials_pass<DT, DIST>(ctx, cur.s, cur.s.elem_offset + i0, cur.s.elem_offset + i1, p.arena);
+      exact_specials_pass<DT, DIST>(cx, d.s, d.s.elem_offset + i0, d.s.elem_offset + i1, p.arena);
     }
-    if (cur.fused) {  // uniform: the spec's exact-count edits inside this CTA's range
+    if (d.fused) {  // uniform: the spec's exact-count edits inside this CTA's range
       __syncthreads();
-      fused_edits<DT, DIST>(ctx, cur.s, cur.s.elem_offset + i0, cur.s.elem_offset + i1, p.arena);
+      fused_edits<DT, DIST>(cx, d.s, d.s.elem_offset + i0, d.s.elem_offset + i1, p.arena);
     }
+    slot ^= 1;
   }
 }
 
