@@ -459,7 +459,8 @@ __global__ void __launch_bounds__(kThreads) fixup_kernel(const __grid_constant__
 // dot-like values: persistent CTAs, each a contiguous run of 64 x 128 output
 // tiles (row-block major, so consecutive tiles share their A rows).  The
 // factors stream through a ring of kDotStages shared-memory slots, one
-// 32-deep k chunk of A (64 rows x 32, row-major) and B (32 x 128) per slot,
+// kDotK-deep k chunk of A (64 rows x kDotK, row-major) and B (kDotK x 128) per
+// slot (64 deep, 2 slots: a whole K = 64 tile per slot, one barrier per tile),
 // filled by cp.async while earlier chunks are multiplied; every output is the
 // k-ascending chain of fused multiply-adds over exactly its K steps.  Thread
 // layout: warp w owns rows 8w..8w+7 of the tile, lane l columns 4l..4l+3 (one
@@ -467,7 +468,7 @@ __global__ void __launch_bounds__(kThreads) fixup_kernel(const __grid_constant__
 // output stores are contiguous.
 // ---------------------------------------------------------------------------
 #ifndef SV_DOT_STAGES
-#define SV_DOT_STAGES 3
+#define SV_DOT_STAGES 2
 #endif
 #ifndef SV_DOT_MINB
 #define SV_DOT_MINB 2
@@ -476,7 +477,7 @@ __global__ void __launch_bounds__(kThreads) fixup_kernel(const __grid_constant__
 #define SV_DOT_THREADS 256  // threads per CTA: one warp per 8 rows of the tile
 #endif
 #ifndef SV_DOT_K
-#define SV_DOT_K 32  // k depth of one shared-memory slot (a multiple of 16)
+#define SV_DOT_K 64  // k depth of one shared-memory slot (a multiple of 16)
 #endif
 constexpr int kDotThreads = SV_DOT_THREADS;
 constexpr int kDotRows = kDotThreads / 32 * 8, kDotCols = 128, kDotK = SV_DOT_K, kDotStages = SV_DOT_STAGES;
