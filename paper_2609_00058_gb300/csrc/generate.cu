@@ -482,6 +482,10 @@ __global__ void __launch_bounds__(kThreads) fixup_kernel(const __grid_constant__
 constexpr int kDotThreads = SV_DOT_THREADS;
 constexpr int kDotRows = kDotThreads / 32 * 8, kDotCols = 128, kDotK = SV_DOT_K, kDotStages = SV_DOT_STAGES;
 static_assert(kDotThreads % 32 == 0 && kDotK % 16 == 0, "dot-like tile shape");
+// every thread issues the same number of copies and together they cover a slot
+static_assert(kDotThreads % (kDotK / 4) == 0 && (kDotRows * kDotK / 4) % kDotThreads == 0 &&
+                  kDotThreads % kDotK == 0 && (kDotK * kDotCols / 4) % kDotThreads == 0,
+              "dot-like slot copies");
 constexpr int kDotSlotFloats = kDotRows * kDotK + kDotK * kDotCols;
 constexpr size_t kDotSmem = (size_t)kDotStages * kDotSlotFloats * sizeof(float);
 
@@ -659,14 +663,20 @@ __global__ void __launch_bounds__(kDotThreads, SV_DOT_MINB) dot_kernel(const __g
 
 // ---------------------------------------------------------------------------
 // the Box-Muller step alone, on caller words (syn_box_muller): pair i of
-// words gives the two normals the generator makes from the same words
+// words gives the two normals the generator makes from the same words.
+// Pairs 2j and 2j + 1 go through box_muller4 together, as the generator's
+// pairs do (an odd last pair is taken twice and stored once).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) box_muller_kernel(const uint2* w, uint64_t n_pairs, float2* z) {
-  for (uint64_t i = (uint64_t)blockIdx.x * kThreads + threadIdx.x; i < n_pairs; i += (uint64_t)gridDim.x * kThreads) {
-    const uint2 p = w[i];
-    float z0, z1;
-    box_muller(p.x, p.y, z0, z1);
-    z[i] = make_float2(z0, z1);
+  const uint64_t n2 = (n_pairs + 1) / 2;
+  for (uint64_t j = (uint64_t)blockIdx.x * kThreads + threadIdx.x; j < n2; j += (uint64_t)gridDim.x * kThreads) {
+    const uint64_t i = 2 * j;
+    const bool two = i + 1 < n_pairs;
+    const uint2 a = w[i], b = two ? w[i + 1] : a;
+    float v[4];
+    box_muller4(make_uint4(a.x, a.y, b.x, b.y), v);
+    z[i] = make_float2(v[0], v[1]);
+    if (two) z[i + 1] = make_float2(v[2], v[3]);
   }
 }
 
@@ -731,7 +741,7 @@ static cudaError_t launch_dot(const DotParams& dp, uint64_t tiles, cudaStream_t 
 cudaError_t launch_box_muller(const uint32_t* words, uint64_t n_pairs, float* z, cudaStream_t st) {
   if (n_pairs == 0) return cudaSuccess;
   const void* fn = reinterpret_cast<const void*>(box_muller_kernel);
-  const uint64_t blocks = std::min<uint64_t>((n_pairs + kThreads - 1) / kThreads, grid_cap_for(fn));
+  const uint64_t blocks = std::min<uint64_t>(((n_pairs + 1) / 2 + kThreads - 1) / kThreads, grid_cap_for(fn));
   box_muller_kernel<<<(unsigned)blocks, launch_block(), 0, st>>>(reinterpret_cast<const uint2*>(words), n_pairs,
                                                             reinterpret_cast<float2*>(z));
   count_launch();

@@ -83,3 +83,19 @@ def test_same_values_as_the_generator(dev):
     gen = a.cpu().numpy().view(np.float32)
     # the generator adds mu = 0 to sigma * z, which turns -0 into +0
     assert np.array_equal(got, gen) and np.array_equal(got[got != 0].view(np.uint32), gen[gen != 0].view(np.uint32))
+
+
+@pytest.mark.parametrize("n_pairs", [1, 7, 1001])
+def test_odd_pair_counts(dev, n_pairs):
+    # pairs go through the transform two at a time; an odd last pair is
+    # taken alone and nothing is written past it
+    import torch
+    rng = np.random.default_rng(n_pairs)
+    words = rng.integers(0, 1 << 32, 2 * n_pairs, dtype=np.uint64).astype(np.uint32)
+    w = torch.from_numpy(words.view(np.int32)).to(dev)
+    out = torch.full((2 * n_pairs + 2,), 7.0, dtype=torch.float32, device=dev)
+    sv.box_muller(w, out=out[:2 * n_pairs])
+    got = out.cpu().numpy()
+    assert np.array_equal(got[2 * n_pairs:], np.full(2, 7.0, np.float32))
+    d = ulp_dist(got[:2 * n_pairs], oracle.box_muller(words))
+    assert d.max() <= 4

@@ -321,6 +321,52 @@ def test_dotlike_chunked(dev):
     assert np.array_equal(g1, h1)
 
 
+@pytest.mark.parametrize("dtype,rows,cols,k", [
+    ("bf16", 1031, 4108, 68),  # two k chunks per tile (64 + 4), ragged rows and columns
+    ("f16", 1100, 4100, 37),   # K % 4 != 0: 4-byte factor copies; many tiles per CTA
+    ("f32", 130, 260, 16),     # a chunk shorter than 64: the held tile's noise runs without FMAs beside it
+    ("bf16", 300, 1032, 64),   # the bench shape's K: one 64-deep chunk per tile
+])
+def test_dotlike_noisy_twin_shapes(dev, dtype, rows, cols, k):
+    """The relative-noise twin, which the kernel makes while it multiplies the
+    next tile: the reference equals the oracle's bit for bit, the twin is
+    within the Box-Muller bound of the oracle's, and it is bit-identical to
+    the twin made afterwards from the stored reference (from_arena); a chunk
+    that starts and ends inside rows writes the same bytes as the whole."""
+    import torch
+    sz = W.DTYPE_BYTES[dtype]
+    n = rows * cols
+    ar = W.Arena()
+    ao, bo = ar.take(4 * rows * k), ar.take(4 * k * cols)
+    ro, co, to = ar.take(sz * n), ar.take(sz * n), ar.take(sz * n)
+    fa = W.GenSpec("f32", "uniform", rows * k, seed=7, stream=0, ref_offset=ao, p0=-1, p1=1)
+    fb = W.GenSpec("f32", "uniform", k * cols, seed=7, stream=1, ref_offset=bo, p0=-1, p1=1)
+    noise = W.Perturb("rel_noise", stream=3, value=2.0 ** -9)
+    d = W.GenSpec(dtype, "dotlike", n, seed=7, stream=2, ref_offset=ro, cand_offset=co, rows=rows, cols=cols,
+                  dot_k=k, a_offset=ao, b_offset=bo, specials=("nan", "pinf", "zero"), special_rate=1e-3,
+                  pelem=noise)
+    g, h = gen_both(dev, [[fa, fb], [d]], ar.size)
+    assert np.array_equal(_view(g, ro, dtype, n), _view(h, ro, dtype, n))
+    check_spec_outputs(g, h, d)
+    a = to_dev(g, dev)
+    twin = W.GenSpec(dtype, "from_arena", n, seed=7, stream=2, ref_offset=None, cand_offset=to, a_offset=ro,
+                     pelem=noise)
+    sv.generate([twin], a)
+    out = a.cpu().numpy()
+    assert np.array_equal(out[co: co + sz * n], out[to: to + sz * n])
+    off = (3 * cols + 8) // 8 * 8  # inside row 3; 16-byte output offsets for every type
+    m = n - off - 7
+    part = d.replace(n=m, elem_offset=off, logical_n=n, ref_offset=ro + off * sz, cand_offset=co + off * sz)
+    b = torch.zeros(ar.size, dtype=torch.uint8, device=dev)
+    sv.generate([fa, fb], b)
+    sv.generate([part], b)
+    got = b.cpu().numpy()
+    for base in (ro, co):
+        lo_b, hi_b = base + off * sz, base + (off + m) * sz
+        assert np.array_equal(got[lo_b: hi_b], g[lo_b: hi_b])
+        assert not got[base: lo_b].any() and not got[hi_b: base + sz * n].any()
+
+
 def test_zero_length_and_single_element(dev):
     specs = [W.GenSpec("f32", "uniform", 0, ref_offset=0, p0=0, p1=1),
              W.GenSpec("i64", "permutation", 1, ref_offset=256, cand_offset=512),
