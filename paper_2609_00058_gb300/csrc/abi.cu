@@ -396,6 +396,17 @@ static void build_pair_plan(const vc_pair* pairs, int n_pairs, Tab& tab, std::ve
   uint64_t slot_base = 0;
   for (Group& g : groups) {
     if (g.key == kSmallKey) {  // one slot each; the combine reads just slot0
+      // the warps start in table order: largest segments first (by the
+      // power of two of their vector count, a stable linear pass), so that
+      // the longest ones do not start last
+      std::vector<int> by_size;
+      by_size.reserve((size_t)(g.end - g.begin));
+      for (int b = 11; b >= 0; --b)
+        for (int k = g.begin; k < g.end; ++k) {
+          const uint64_t v = cmp_vectors(pairs[order[k]]);
+          if ((v == 0 ? 0 : 64 - __builtin_clzll(v)) == b) by_size.push_back(order[k]);
+        }
+      std::copy(by_size.begin(), by_size.end(), order.begin() + g.begin);
       for (int k = g.begin; k < g.end; ++k) {
         DevPair& d = tab[k];
         d.p = pairs[order[k]];
@@ -446,7 +457,7 @@ static int run_pair_plan(const DevPair* host, const DevPair* dev, int n_pairs, c
 // the plan of one syn_generate: the spec table grouped by dtype x
 // distribution (stable), each group's weighted units and launch shape, every
 // spec's first unit, and its exact-count fixup threads -- edits are applied by
-// the generating CTAs where a CTA's slice (at most 4 x chunk elements) meets
+// the generating warps where a warp's slice (at most 4 x chunk elements) meets
 // few strata, else by the fixup kernel.  Returns the fixup threads.
 template <class Tab>
 static uint64_t build_spec_plan(const syn_spec* specs, int n_specs, Tab& tab, std::vector<Group>& groups) {

@@ -411,6 +411,8 @@ __device__ void flush(Acc& a, Partial* out) {
 // one instantiation per dtype; the host groups the pairs by dtype
 template <int DT>
 __global__ void __launch_bounds__(kThreads, 3) cmp_kernel(const __grid_constant__ CmpParams p) {
+  pdl_wait();
+  pdl_trigger();
   if (p.flag && *p.flag >= 0) return;  // an earlier stage failed
   __shared__ uint64_t staged[kStagedStarts];
   const uint64_t u0 = (uint64_t)blockIdx.x * p.chunk;
@@ -455,6 +457,8 @@ __device__ __forceinline__ void warp_segment(const vc_pair& pr, const uint8_t* c
 }
 
 __global__ void __launch_bounds__(kThreads) cmp_small_kernel(const __grid_constant__ CmpParams p) {
+  pdl_wait();
+  pdl_trigger();
   const int w = (int)(blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5)), lane = threadIdx.x & 31;
   if (w >= p.n) return;
   const DevPair* dp = pentry(p, w);
@@ -531,6 +535,8 @@ __device__ __forceinline__ vc_result skipped_result() {
 }
 
 __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant__ CombParams p) {
+  pdl_wait();
+  pdl_trigger();
   const int e = (int)((blockIdx.x * (uint64_t)kThreads + threadIdx.x) >> 5);
   const int lane = threadIdx.x & 31;
   if (e >= p.n) return;
@@ -545,6 +551,8 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const __grid_constant
 // the failing stage so that later groups do not run.  Stages of a group are
 // compared in one pass; the verdicts equal those of running them one by one.
 __global__ void __launch_bounds__(kThreads) combine_stages_kernel(const __grid_constant__ CombParams p) {
+  pdl_wait();
+  pdl_trigger();
   __shared__ vc_result res[SV_INLINE_ENTRIES];
   const int e = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (!p.first_group && *p.flag >= 0) {  // an earlier group failed: nothing of this group ran
@@ -922,16 +930,17 @@ cudaError_t launch_compare_group(uint32_t dtype, const DevPair* host, const DevP
   cp.ref = ref;
   cp.partials = partials;
   cp.flag = flag;
+  cudaError_t e;
   switch (dtype) {
-    case SV_F32: cmp_kernel<SV_F32><<<sh.grid, launch_block(), 0, st>>>(cp); break;
-    case SV_F16: cmp_kernel<SV_F16><<<sh.grid, launch_block(), 0, st>>>(cp); break;
-    case SV_BF16: cmp_kernel<SV_BF16><<<sh.grid, launch_block(), 0, st>>>(cp); break;
-    case SV_I32: cmp_kernel<SV_I32><<<sh.grid, launch_block(), 0, st>>>(cp); break;
-    case SV_I64: cmp_kernel<SV_I64><<<sh.grid, launch_block(), 0, st>>>(cp); break;
-    default: cmp_kernel<SV_U32><<<sh.grid, launch_block(), 0, st>>>(cp); break;
+    case SV_F32: e = launch_chained(cmp_kernel<SV_F32>, sh.grid, launch_block(), st, cp); break;
+    case SV_F16: e = launch_chained(cmp_kernel<SV_F16>, sh.grid, launch_block(), st, cp); break;
+    case SV_BF16: e = launch_chained(cmp_kernel<SV_BF16>, sh.grid, launch_block(), st, cp); break;
+    case SV_I32: e = launch_chained(cmp_kernel<SV_I32>, sh.grid, launch_block(), st, cp); break;
+    case SV_I64: e = launch_chained(cmp_kernel<SV_I64>, sh.grid, launch_block(), st, cp); break;
+    default: e = launch_chained(cmp_kernel<SV_U32>, sh.grid, launch_block(), st, cp); break;
   }
   count_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 cudaError_t launch_compare_small(const DevPair* host, const DevPair* dev, int n, const uint8_t* cand,
@@ -946,9 +955,9 @@ cudaError_t launch_compare_small(const DevPair* host, const DevPair* dev, int n,
   cp.partials = partials;
   cp.flag = nullptr;
   const unsigned blocks = (unsigned)((n + kThreads / 32 - 1) / (kThreads / 32));
-  cmp_small_kernel<<<blocks, launch_block(), 0, st>>>(cp);
+  const cudaError_t e = launch_chained(cmp_small_kernel, blocks, launch_block(), st, cp);
   count_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const Partial* partials,
@@ -960,15 +969,16 @@ cudaError_t launch_combine(const DevPair* host, const DevPair* dev, int n, const
   cp.results = results;
   cp.flag = flag;
   cp.first_group = first_group;
+  cudaError_t e;
   if (flag) {  // a progressive group: one CTA, stages in order
     if (n > SV_INLINE_ENTRIES || dev) return cudaErrorInvalidValue;
-    combine_stages_kernel<<<1, launch_block(), 0, st>>>(cp);
+    e = launch_chained(combine_stages_kernel, 1u, launch_block(), st, cp);
   } else {
     const uint64_t blocks = ((uint64_t)n * 32 + kThreads - 1) / kThreads;
-    combine_kernel<<<(unsigned)blocks, launch_block(), 0, st>>>(cp);
+    e = launch_chained(combine_kernel, (unsigned)blocks, launch_block(), st, cp);
   }
   count_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 }  // namespace sv

@@ -320,6 +320,8 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
 // that a launch only sees its own kind
 template <int DT, int DIST>
 __global__ void __launch_bounds__(kThreads, SV_GEN_MINB) gen_kernel(const __grid_constant__ GenParams p) {
+  pdl_wait();
+  pdl_trigger();
   // two slots for the entry in use and its context: an entry is staged into
   // the slot its predecessor did not use, so one barrier per entry suffices
   // (a slot's previous user is two entries back, which every thread finished
@@ -447,6 +449,8 @@ __device__ void fix_dispatch(const Ctx& c, const syn_spec& s, uint64_t u, uint8_
 }
 
 __global__ void __launch_bounds__(kThreads) fixup_kernel(const __grid_constant__ GenParams p) {
+  pdl_wait();
+  pdl_trigger();
   const uint64_t u = (uint64_t)blockIdx.x * kThreads + threadIdx.x;
   if (u >= p.total) return;
   const DevSpec* e = entry(p, find_fix_entry(p, u));
@@ -703,15 +707,16 @@ cudaError_t launch_generate_group(uint32_t dtype, uint32_t dist, const DevSpec* 
   gp.total = units;
   gp.chunk = sh.chunk;
   gp.arena = arena;
+  cudaError_t e = cudaSuccess;
   switch (SV_COMBO(dtype, dist)) {
 #define SV_CASE(DT, DIST) \
-  case SV_COMBO(DT, DIST): gen_kernel<DT, DIST><<<sh.grid, launch_block(), 0, st>>>(gp); break;
+  case SV_COMBO(DT, DIST): e = launch_chained(gen_kernel<DT, DIST>, sh.grid, launch_block(), st, gp); break;
     SV_GEN_COMBOS(SV_CASE)
 #undef SV_CASE
     default: return cudaErrorInvalidValue;
   }
   count_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_t total_units, uint8_t* arena,
@@ -723,9 +728,9 @@ cudaError_t launch_fixup(const DevSpec* host, const DevSpec* dev, int n, uint64_
   gp.chunk = 0;
   gp.arena = arena;
   const uint64_t blocks = (total_units + kThreads - 1) / kThreads;
-  fixup_kernel<<<(unsigned)blocks, launch_block(), 0, st>>>(gp);
+  const cudaError_t e = launch_chained(fixup_kernel, (unsigned)blocks, launch_block(), st, gp);
   count_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 template <int DT, bool A16>

@@ -82,6 +82,28 @@ LaunchShape shape_for(uint64_t units, uint64_t tiles, uint32_t cap, uint64_t ali
 // SMs x resident CTAs of this kernel at `block` threads per CTA (cached per
 // device), at most kGridCap
 uint32_t grid_cap_for(const void* kernel, size_t dyn_smem = 0, int block = kThreads);
+// a launch in a chain of this library's kernels (programmatic dependent
+// launch, sm_90+): the kernel may be scheduled while the previous kernel of
+// the stream still runs, so its launch latency and ramp overlap that
+// kernel's tail; it starts with pdl_wait() (griddepcontrol.wait), which
+// returns once the previous kernel has completed and its stores are visible,
+// so no data dependency changes.  Errors as for <<<>>>.
+template <typename P>
+inline cudaError_t launch_chained(void (*kernel)(P), unsigned grid, unsigned block, cudaStream_t st, const P& p) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, p);
+  const cudaError_t last = cudaGetLastError();  // clears what the launch left
+  return e != cudaSuccess ? e : last;
+}
 // one more kernel launched by this library (the sv_kernel_launches counter)
 void count_launch();
 // the block size of every launch: kThreads, or 0 (an invalid configuration,

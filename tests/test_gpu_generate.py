@@ -527,3 +527,41 @@ def test_generate_plan_equals_syn_generate(dev, n_specs):
         b = torch.zeros(ar.size, dtype=torch.uint8, device=dev)
         plan(b)
         assert torch.equal(a, b)
+
+
+
+@pytest.mark.parametrize("n_specs", [40, 300])
+def test_plan_mixed_kinds(dev, n_specs):
+    """A plan over many specs of every size class writes the bytes of
+    syn_generate: arena-source twins, exact-count specials, fused and fixup
+    edits, element-wise perturbations."""
+    import torch
+    ar = W.Arena()
+    src_n = 70000
+    src = ar.take(2 * src_n)
+    kinds = [dict(dtype="f32", dist="normal", p0=0.0, p1=1.0, specials=("nan", "ninf"), special_rate=1e-3,
+                  special_exact=True),
+             dict(dtype="f16", dist="from_arena", a_offset=src, pelem=W.Perturb("rel_noise", stream=3, value=2.0 ** -9)),
+             dict(dtype="i32", dist="int_range", i0=-9, i1=9, pcount=W.Perturb("count_add", stream=5, count=2, ivalue=1)),
+             dict(dtype="bf16", dist="uniform", p0=-3.0, p1=3.0, pelem=W.Perturb("rate_add_pm", stream=6, rate=0.01,
+                                                                                  value=0.5)),
+             dict(dtype="i64", dist="permutation", pcount=W.Perturb("swap_pairs", stream=4, count=3))]
+    specs = []
+    for i in range(n_specs):
+        kw = kinds[i % len(kinds)]
+        n = [1, 7, 100, 8192, 20001, 65536][i % 6]
+        if "pcount" in kw:
+            n = max(n, 16)  # room for the edits' strata
+        sz = W.DTYPE_BYTES[kw["dtype"]]
+        specs.append(W.GenSpec(n=n, seed=i, stream=i, ref_offset=ar.take(n * sz), cand_offset=ar.take(n * sz), **kw))
+    g = torch.Generator(device=dev)
+    g.manual_seed(n_specs)
+    base = torch.zeros(ar.size, dtype=torch.uint8, device=dev)
+    base[src: src + 2 * src_n] = (torch.randn(src_n, device=dev, generator=g) * 4).half().view(torch.uint8)
+    a = base.clone()
+    sv.generate(specs, a)
+    plan = sv.GeneratePlan(specs, ar.size, device=dev)
+    for _ in range(2):
+        b = base.clone()
+        plan(b)
+        assert torch.equal(a, b)
