@@ -60,18 +60,18 @@ NCU_TRAFFIC = {
     # one single-pass launch list per workload (python bench.py --workload W
     # --only-headline --steps 2 --warmup 1 --no-cpu-baseline): the step's own
     # launches of each role, summed over its 7 steps and divided by 7
-    ("perm_i64", "generate", "adc8ab0ad9574e56"): 4234475886,  # gen_kernel<i64, permutation>, edits fused
-    ("perm_i64", "verify", "e6a8a19b21a7816d"): 4295353454,    # cmp_kernel<i64> + combine_kernel
-    ("ladder", "generate", "adc8ab0ad9574e56"): 1316507246,    # gen_kernel<f32, normal>, one launch
-    ("ladder", "verify", "e6a8a19b21a7816d"): 36023881,        # 3 stage groups: cmp_kernel + combine_stages_kernel
-    ("dotlike_bf16", "generate", "adc8ab0ad9574e56"): 4435823141,  # factors gen_kernel + dot_kernel<bf16>
-    ("dotlike_bf16", "verify", "e6a8a19b21a7816d"): 4298318811,    # cmp_kernel<bf16> + combine_kernel
+    ("perm_i64", "generate", "50ebf9c04acc3258"): 4234279570,  # gen_kernel<i64, permutation>, edits fused
+    ("perm_i64", "verify", "76cd7526f78a111f"): 4295220224,    # cmp_kernel<i64> + combine_kernel
+    ("ladder", "generate", "50ebf9c04acc3258"): 1316649984,    # gen_kernel<f32, normal>, one launch
+    ("ladder", "verify", "76cd7526f78a111f"): 36021870,        # 3 stage groups: cmp_kernel + combine_stages_kernel
+    ("dotlike_bf16", "generate", "50ebf9c04acc3258"): 4437972736,  # factors gen_kernel + dot_kernel<bf16>
+    ("dotlike_bf16", "verify", "76cd7526f78a111f"): 4298131858,    # cmp_kernel<bf16> + combine_kernel
     # the two small workloads' outputs stay in L2 through the step (DRAM
     # counts only what the caches write back meanwhile)
-    ("segmented", "generate", "adc8ab0ad9574e56"): 5589614,
-    ("segmented", "verify", "e6a8a19b21a7816d"): 146431817,
-    ("fp32_pair", "generate", "adc8ab0ad9574e56"): 77166,
-    ("fp32_pair", "verify", "e6a8a19b21a7816d"): 8449317,
+    ("segmented", "generate", "50ebf9c04acc3258"): 5650286,
+    ("segmented", "verify", "76cd7526f78a111f"): 146438619,
+    ("fp32_pair", "generate", "50ebf9c04acc3258"): 90441,
+    ("fp32_pair", "verify", "76cd7526f78a111f"): 8450743,
 }
 ROLE_SOURCES = {"generate": ("generate.cu", "sv_device.cuh", "sv_kernels.h"),
                 "verify": ("compare.cu", "sv_device.cuh", "sv_kernels.h")}
