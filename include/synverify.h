@@ -22,7 +22,11 @@
  *   and copied to the workspace with cudaMemcpyAsync; a staging buffer is
  *   reused only after the copy issued from it has completed.  (If no staging
  *   buffer can be had, the table goes from ordinary host memory, and the
- *   driver may then wait for the stream before that copy.)
+ *   driver may then wait for the stream before that copy.)  The generator,
+ *   compare and combine kernels are launched as programmatic dependent
+ *   launches: one may be scheduled while the previous kernel of the stream
+ *   still runs, and it waits on the device for that kernel to complete before
+ *   it reads or writes memory, so stream order holds as for plain launches.
  * - Errors: 0 on success, a negative SV_E* status otherwise.  All arguments are
  *   validated on the host before anything is enqueued, so a validation error
  *   leaves device memory untouched.  SV_ECUDA reports a CUDA launch or copy
