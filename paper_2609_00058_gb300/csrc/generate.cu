@@ -669,18 +669,25 @@ __global__ void __launch_bounds__(kDotThreads, SV_DOT_MINB) dot_kernel(const __g
 // the Box-Muller step alone, on caller words (syn_box_muller): pair i of
 // words gives the two normals the generator makes from the same words.
 // Pairs 2j and 2j + 1 go through box_muller4 together, as the generator's
-// pairs do (an odd last pair is taken twice and stored once).
+// pairs do; an odd last pair goes through the single-pair box_muller, whose
+// values the packed form reproduces bit for bit.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) box_muller_kernel(const uint2* w, uint64_t n_pairs, float2* z) {
   const uint64_t n2 = (n_pairs + 1) / 2;
   for (uint64_t j = (uint64_t)blockIdx.x * kThreads + threadIdx.x; j < n2; j += (uint64_t)gridDim.x * kThreads) {
     const uint64_t i = 2 * j;
-    const bool two = i + 1 < n_pairs;
-    const uint2 a = w[i], b = two ? w[i + 1] : a;
-    float v[4];
-    box_muller4(make_uint4(a.x, a.y, b.x, b.y), v);
-    z[i] = make_float2(v[0], v[1]);
-    if (two) z[i + 1] = make_float2(v[2], v[3]);
+    const uint2 a = w[i];
+    if (i + 1 < n_pairs) {
+      const uint2 b = w[i + 1];
+      float v[4];
+      box_muller4(make_uint4(a.x, a.y, b.x, b.y), v);
+      z[i] = make_float2(v[0], v[1]);
+      z[i + 1] = make_float2(v[2], v[3]);
+    } else {
+      float z0, z1;
+      box_muller(a.x, a.y, z0, z1);
+      z[i] = make_float2(z0, z1);
+    }
   }
 }
 

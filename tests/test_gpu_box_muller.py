@@ -99,3 +99,21 @@ def test_odd_pair_counts(dev, n_pairs):
     assert np.array_equal(got[2 * n_pairs:], np.full(2, 7.0, np.float32))
     d = ulp_dist(got[:2 * n_pairs], oracle.box_muller(words))
     assert d.max() <= 4
+
+
+def test_packed_pairs_equal_the_single_pair_form(dev):
+    # syn_box_muller runs pairs two at a time through the packed f32x2 steps
+    # and an odd last pair through the single-pair steps: every pair of a
+    # long call, taken again alone (a one-pair call), gives the same bits
+    import torch
+    rng = np.random.default_rng(11)
+    n_pairs = 4096
+    words = rng.integers(0, 1 << 32, 2 * n_pairs, dtype=np.uint64).astype(np.uint32)
+    # include the edge words: u1 = 1 (L = -0), the smallest u1, quarter-turn boundaries
+    words[0:8] = [0xFFFFFF00, 0x00000000, 0x000000FF, 0x40000000, 0xFFFFFFFF, 0x3FFFFF00, 0x12345678, 0xC0000000]
+    w = torch.from_numpy(words.view(np.int32)).to(dev)
+    packed = sv.box_muller(w).cpu().numpy().view(np.uint32)
+    single = np.empty_like(packed)
+    for i in range(n_pairs):
+        single[2 * i: 2 * i + 2] = sv.box_muller(w[2 * i: 2 * i + 2]).cpu().numpy().view(np.uint32)
+    assert np.array_equal(packed, single)
