@@ -77,8 +77,47 @@ __device__ __forceinline__ void store4(uint8_t* base, uint64_t i, const typename
   }
 }
 
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+// one quantum (QB bytes: 8, 16 or 32) from global to shared memory by cp.async;
+// both addresses aligned to min(QB, 16)
+template <int QB>
+__device__ __forceinline__ void copy_quantum_async(uint8_t* dst, const uint8_t* src) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+  if constexpr (QB == 8) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(d), "l"(src) : "memory");
+  } else if constexpr (QB == 16) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(src) : "memory");
+  } else {
+    static_assert(QB == 32, "quantum bytes");
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(src) : "memory");
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d + 16), "l"(src + 16) : "memory");
+  }
+}
+
+// the four elements of a quantum from its bytes (in shared memory)
+template <int DT>
+__device__ __forceinline__ void unpack_quantum(const uint8_t* p, typename Store<DT>::T v[4]) {
+  using T = typename Store<DT>::T;
+  if constexpr (elem_bytes(DT) == 4) {
+    const uint4 w = *reinterpret_cast<const uint4*>(p);
+    v[0] = (T)w.x, v[1] = (T)w.y, v[2] = (T)w.z, v[3] = (T)w.w;
+  } else if constexpr (elem_bytes(DT) == 2) {
+    const uint2 w = *reinterpret_cast<const uint2*>(p);
+    v[0] = (T)(w.x & 0xFFFFu), v[1] = (T)(w.x >> 16), v[2] = (T)(w.y & 0xFFFFu), v[3] = (T)(w.y >> 16);
+  } else {
+    const ulonglong2 a = reinterpret_cast<const ulonglong2*>(p)[0], b = reinterpret_cast<const ulonglong2*>(p)[1];
+    v[0] = (T)a.x, v[1] = (T)a.y, v[2] = (T)b.x, v[3] = (T)b.y;
+  }
+}
+
 #ifndef SV_GEN_MINB
 #define SV_GEN_MINB 2  // resident CTAs per SM the register budget must allow
+#endif
+#ifndef SV_ARENA_RING_BYTES
+#define SV_ARENA_RING_BYTES 64  // shared-memory ring bytes per thread for arena-source quanta
 #endif
 #ifndef SV_GEN_PIPELINE
 #define SV_GEN_PIPELINE 1  // draw the next iteration's VALUE blocks before this iteration's maps (0: after)
@@ -219,24 +258,36 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
   if constexpr (DIST == SV_FROM_ARENA) {
     // values read from memory, two quanta per iteration: their relative noise
     // (the usual perturbation of such twins) runs as two interleaved chains.
-    // The next iteration's source vectors are loaded before this iteration's
-    // arithmetic, so their latency overlaps it.
-    T na[4], nb[4];
-    if (q < qfull) base4<DT, DIST>(c, eo + (q << 2), na);
-    if (q + kThreads < qfull) base4<DT, DIST>(c, eo + ((q + kThreads) << 2), nb);
-    for (; q < qfull; q += 2ull * kThreads) {
+    // The source quanta of the next kArenaAhead iterations are in flight as
+    // cp.async copies into this thread's own slots of a shared-memory ring (no
+    // registers held across the arithmetic, no barrier: a thread reads only
+    // what it copied); iteration i waits for its own copies, reads them, and
+    // after its arithmetic refills its slot with iteration i + kArenaAhead.
+    constexpr int QB = 4 * elem_bytes(DT);  // bytes of a quantum
+    constexpr int kArenaAhead = SV_ARENA_RING_BYTES / (2 * QB) > 0 ? SV_ARENA_RING_BYTES / (2 * QB) : 1;
+    __shared__ __align__(16) uint8_t ring[kArenaAhead * 2 * kThreads * QB];
+    const uint8_t* src = reinterpret_cast<const uint8_t*>(c.A) + eo * elem_bytes(DT);  // 16-byte aligned; quanta on QB
+    const int tid = (int)threadIdx.x;
+    auto slot_of = [&](uint64_t it, int k) { return ring + (((int)(it % kArenaAhead) * 2 + k) * kThreads + tid) * QB; };
+    auto fill = [&](uint64_t it, uint64_t qi) {  // the two quanta of iteration it (qi: its first)
+      if (qi < qfull) copy_quantum_async<QB>(slot_of(it, 0), src + (qi << 2) * elem_bytes(DT));
+      if (qi + kThreads < qfull) copy_quantum_async<QB>(slot_of(it, 1), src + ((qi + kThreads) << 2) * elem_bytes(DT));
+      cp_async_commit();  // one group per iteration, empty past the end: uniform counting
+    };
+#pragma unroll
+    for (int a = 0; a < kArenaAhead; ++a) fill((uint64_t)a, q + 2ull * kThreads * a);
+    for (uint64_t it = 0; q < qfull; q += 2ull * kThreads, ++it) {
       const uint64_t q2 = q + kThreads, ia = q << 2, ib = q2 << 2;
       const bool two = q2 < qfull;
+      cp_async_wait<kArenaAhead - 1>();  // this thread's copies of iteration it have landed
       T va[4], vb[4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) va[j] = na[j], vb[j] = nb[j];
-      const uint64_t qn = q + 2ull * kThreads;
-      if (qn < qfull) base4<DT, DIST>(c, eo + (qn << 2), na);
-      if (qn + kThreads < qfull) base4<DT, DIST>(c, eo + ((qn + kThreads) << 2), nb);
+      unpack_quantum<DT>(slot_of(it, 0), va);
+      if (two) unpack_quantum<DT>(slot_of(it, 1), vb);
       if (c.sp_thr) {
         specials4<DT, DIST>(c, cold, eo + ia, va);
         if (two) specials4<DT, DIST>(c, cold, eo + ib, vb);
       }
+      bool done = false;
       if constexpr (is_float(DT)) {
         if (two && cand && c.pe_kind == SV_PERT_REL_NOISE) {
           if (ref) {
@@ -246,12 +297,16 @@ __device__ void gen_run(const Ctx& cold, const syn_spec& s, uint64_t i0, uint64_
           rel_noise4x2<DT>(c, eo + ia, va, eo + ib, vb);
           store4<DT>(cand, ia, va, 4);
           store4<DT>(cand, ib, vb, 4);
-          continue;
+          done = true;
         }
       }
-      store_quantum<DT>(c, cold, ref, cand, eo + ia, ia, va, 4);
-      if (two) store_quantum<DT>(c, cold, ref, cand, eo + ib, ib, vb, 4);
+      if (!done) {
+        store_quantum<DT>(c, cold, ref, cand, eo + ia, ia, va, 4);
+        if (two) store_quantum<DT>(c, cold, ref, cand, eo + ib, ib, vb, 4);
+      }
+      fill(it + kArenaAhead, q + 2ull * kThreads * kArenaAhead);  // the slot's values are consumed
     }
+    cp_async_wait<0>();
   } else {
     if constexpr (one_block_dist<DT, DIST>()) {
       if (!c.sp_thr) {
@@ -509,9 +564,6 @@ __device__ __forceinline__ void cp_async4(float* dst, const float* src, bool val
   const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(src), "r"(valid ? 4 : 0) : "memory");
 }
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
 
 // position in a CTA's run of (tile, k chunk) steps, advanced without division
 struct DotCursor {
