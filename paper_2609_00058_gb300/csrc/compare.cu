@@ -641,6 +641,17 @@ __device__ __forceinline__ vc_result tile_result(const Partial& q, uint64_t n, b
 #ifndef SV_TILE_U
 #define SV_TILE_U 2  // 16-byte vectors per operand a tile-kernel thread loads per step
 #endif
+#ifndef SV_TILE_GROUP_RING
+#define SV_TILE_GROUP_RING 2  // steps a tile-group lane keeps in flight through its shared-memory ring (0: none)
+#endif
+__device__ __forceinline__ void cp_async16_tile(void* dst, const void* src) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit_tile() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_tile() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
 #ifndef SV_TILE_GROUP_U
 #define SV_TILE_GROUP_U 4  // rows a tile-group lane loads per step (one 16-byte vector per operand each)
 #endif
@@ -665,6 +676,47 @@ __device__ __forceinline__ void tile_group(const TileParams& p, uint64_t item, i
   uint64_t idx = r0 * t.cols + col;
   Acc a;
   acc_reset(a);
+#if SV_TILE_GROUP_RING
+  // the rows of the next kRing steps are in flight as cp.async copies into
+  // this thread's own slots of a shared-memory ring (one 16-byte vector per
+  // operand and row; slot-major with the threads innermost, so a warp's
+  // copies and reads are contiguous): step st waits for its own copies,
+  // reads them and refills its slot with step st + kRing
+  constexpr int kRing = SV_TILE_GROUP_RING;
+  extern __shared__ __align__(16) uint4 tring[];
+  const uint32_t steps = (h + U - 1) / U;
+  auto at = [&](uint32_t st, int u, int op) { return tring + ((int)((st % kRing) * U + u) * 2 + op) * kThreads + threadIdx.x; };
+  auto fill = [&](uint32_t st) {
+    if (st < steps) {
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const uint32_t row = st * U + u;
+        if (row < h) {
+          cp_async16_tile(at(st, u, 0), xp + row * xpb);
+          cp_async16_tile(at(st, u, 1), yp + row * ypb);
+        }
+      }
+    }
+    cp_async_commit_tile();  // one group per step, empty past the end: uniform counting
+  };
+#pragma unroll
+  for (int s0 = 0; s0 < kRing; ++s0) fill((uint32_t)s0);
+  for (uint32_t st = 0, r = 0; r < h; ++st, r += U) {  // h is the same for every lane
+    cp_async_wait_tile<kRing - 1>();
+    uint4 x[U], y[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (r + u < h) {
+        x[u] = *at(st, u, 0);
+        y[u] = *at(st, u, 1);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (r + u < h) do_vector<DT>(a, tol, x[u], y[u], idx + (uint64_t)u * t.cols);
+    idx += U * t.cols;
+    fill(st + kRing);  // the slot's values are in registers
+#else
   for (uint32_t r = 0; r < h; r += U) {  // h is the same for every lane
     uint4 x[U], y[U];
 #pragma unroll
@@ -680,12 +732,16 @@ __device__ __forceinline__ void tile_group(const TileParams& p, uint64_t item, i
     xp += U * xpb;
     yp += U * ypb;
     idx += U * t.cols;
+#endif
     if constexpr (is_float(DT)) {
       float m = a.maxrel_f;
       for (int o = vr >> 1; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
       a.relthr = m;
     }
   }
+#if SV_TILE_GROUP_RING
+  cp_async_wait_tile<0>();
+#endif
   const Partial f = warp_fold<is_float(DT)>(a, vr);
   if (lane % vr == 0)
     p.results[ti * p.ntc + gj * p.G + (uint64_t)(lane / vr)] = tile_result(f, (uint64_t)h * t.tile_cols, is_float(DT));
@@ -813,14 +869,17 @@ static const void* tile_group_kernel_for(uint32_t dtype) {
   }
 }
 
+// dynamic shared memory of a tile-group CTA: its threads' rings
+constexpr size_t kTileRingSmem = (size_t)SV_TILE_GROUP_RING * SV_TILE_GROUP_U * 2 * kThreads * 16;
+
 static void launch_tile_groups(const TileParams& tp, uint32_t grid, cudaStream_t st) {
   switch (tp.t.dtype) {
-    case SV_F32: tile_group_kernel<SV_F32><<<grid, launch_block(), 0, st>>>(tp); break;
-    case SV_F16: tile_group_kernel<SV_F16><<<grid, launch_block(), 0, st>>>(tp); break;
-    case SV_BF16: tile_group_kernel<SV_BF16><<<grid, launch_block(), 0, st>>>(tp); break;
-    case SV_I32: tile_group_kernel<SV_I32><<<grid, launch_block(), 0, st>>>(tp); break;
-    case SV_I64: tile_group_kernel<SV_I64><<<grid, launch_block(), 0, st>>>(tp); break;
-    default: tile_group_kernel<SV_U32><<<grid, launch_block(), 0, st>>>(tp); break;
+    case SV_F32: tile_group_kernel<SV_F32><<<grid, launch_block(), kTileRingSmem, st>>>(tp); break;
+    case SV_F16: tile_group_kernel<SV_F16><<<grid, launch_block(), kTileRingSmem, st>>>(tp); break;
+    case SV_BF16: tile_group_kernel<SV_BF16><<<grid, launch_block(), kTileRingSmem, st>>>(tp); break;
+    case SV_I32: tile_group_kernel<SV_I32><<<grid, launch_block(), kTileRingSmem, st>>>(tp); break;
+    case SV_I64: tile_group_kernel<SV_I64><<<grid, launch_block(), kTileRingSmem, st>>>(tp); break;
+    default: tile_group_kernel<SV_U32><<<grid, launch_block(), kTileRingSmem, st>>>(tp); break;
   }
 }
 
@@ -878,7 +937,7 @@ cudaError_t launch_compare_tiles(const vc_tiles& t, uint64_t ntc, uint64_t n_til
     }
     if (tp.n_groups) {  // the groups, then the other tiles one warp each
       const uint64_t want = (tp.n_groups + kThreads / 32 - 1) / (kThreads / 32);
-      launch_tile_groups(tp, (uint32_t)umin(want, grid_cap_for(tile_group_kernel_for(t.dtype))), st);
+      launch_tile_groups(tp, (uint32_t)umin(want, grid_cap_for(tile_group_kernel_for(t.dtype), kTileRingSmem)), st);
       count_launch();
     }
     const uint64_t rest = n_tiles - tp.n_groups * tp.G;
