@@ -60,18 +60,18 @@ NCU_TRAFFIC = {
     # one single-pass launch list per workload (python bench.py --workload W
     # --only-headline --steps 2 --warmup 1 --no-cpu-baseline): the step's own
     # launches of each role, summed over its 7 steps and divided by 7
-    ("perm_i64", "generate", "1c4f4b4c9fb23b7d"): 4234284105,  # gen_kernel<i64, permutation>, edits fused
-    ("perm_i64", "verify", "76cd7526f78a111f"): 4295303826,    # cmp_kernel<i64> + combine_kernel
-    ("ladder", "generate", "1c4f4b4c9fb23b7d"): 1316533541,    # gen_kernel<f32, normal>, one launch
-    ("ladder", "verify", "76cd7526f78a111f"): 36022162,        # 3 stage groups: cmp_kernel + combine_stages_kernel
-    ("dotlike_bf16", "generate", "1c4f4b4c9fb23b7d"): 4439732041,  # factors gen_kernel + dot_kernel<bf16>
-    ("dotlike_bf16", "verify", "76cd7526f78a111f"): 4298143415,    # cmp_kernel<bf16> + combine_kernel
+    ("perm_i64", "generate", "1c4f4b4c9fb23b7d"): 4234255799,  # gen_kernel<i64, permutation>, edits fused
+    ("perm_i64", "verify", "792e3c49e8acd81c"): 4295342738,    # cmp_kernel<i64> + combine_kernel
+    ("ladder", "generate", "1c4f4b4c9fb23b7d"): 1316475611,    # gen_kernel<f32, normal>, one launch
+    ("ladder", "verify", "792e3c49e8acd81c"): 36022930,        # 3 stage groups: cmp_kernel + combine_stages_kernel
+    ("dotlike_bf16", "generate", "1c4f4b4c9fb23b7d"): 4442408814,  # factors gen_kernel + dot_kernel<bf16>
+    ("dotlike_bf16", "verify", "792e3c49e8acd81c"): 4298158373,    # cmp_kernel<bf16> + combine_kernel
     # the two small workloads' outputs stay in L2 through the step (DRAM
     # counts only what the caches write back meanwhile)
-    ("segmented", "generate", "1c4f4b4c9fb23b7d"): 5668827,
-    ("segmented", "verify", "76cd7526f78a111f"): 146442240,
-    ("fp32_pair", "generate", "1c4f4b4c9fb23b7d"): 91941,
-    ("fp32_pair", "verify", "76cd7526f78a111f"): 8450158,
+    ("segmented", "generate", "1c4f4b4c9fb23b7d"): 5694427,
+    ("segmented", "verify", "792e3c49e8acd81c"): 146442240,
+    ("fp32_pair", "generate", "1c4f4b4c9fb23b7d"): 90514,
+    ("fp32_pair", "verify", "792e3c49e8acd81c"): 8452718,
 }
 ROLE_SOURCES = {"generate": ("generate.cu", "sv_device.cuh", "sv_kernels.h"),
                 "verify": ("compare.cu", "sv_device.cuh", "sv_kernels.h")}
