@@ -108,3 +108,41 @@ def test_random_tables_match_the_oracle(dev, seed):
         sv.GeneratePlan(call, size, device=dev)(a)
     torch.cuda.synchronize()
     assert np.array_equal(a.cpu().numpy(), g)
+
+
+def random_pairs(rng, n_pairs):
+    """A table of pairs of random dtypes, sizes (empty, ragged, below and above
+    the small-segment limit), tolerances and NaN rules over one arena of
+    planted near and far mismatches and non-finite patterns."""
+    ar = W.Arena()
+    pairs, chunks = [], []
+    for i in range(n_pairs):
+        dt = str(rng.choice(["f32", "f16", "bf16", "i32", "u32", "i64"]))
+        n = int(rng.choice([0, 1, 5, 8, 64, 1000, 4096, 16383, 20000, 70001]))
+        c, r = W.random_pair_arrays(dt, max(n, 1), seed=int(rng.integers(0, 1 << 30)),
+                                    mismatch_frac=float(rng.choice([0.0, 1e-3, 0.05])))
+        sz = W.DTYPE_BYTES[dt]
+        co, ro = ar.take(n * sz), ar.take(n * sz)
+        chunks += [(co, c[:n * sz]), (ro, r[:n * sz])]
+        atol, rtol = (float(rng.choice([0.0, 1e-6, 1e-3, 0.5])), float(rng.choice([0.0, 1e-5, 1e-2])))
+        pairs.append(W.Pair(dt, n, co, ro, atol=atol, rtol=rtol, equal_nan=bool(rng.random() < 0.8)))
+    buf = np.zeros(ar.size, np.uint8)
+    for off, data in chunks:
+        buf[off: off + data.size] = data
+    return pairs, buf
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_random_pair_tables_match_the_oracle(dev, seed):
+    import oracle
+    import torch
+    from gpu_util import assert_results_match
+    rng = np.random.default_rng(5000 + seed)
+    pairs, buf = random_pairs(rng, int(rng.choice([3, 40, 300])))
+    a = torch.from_numpy(buf).to(dev)
+    want = oracle.compare(pairs, buf, buf)
+    got = sv.decode_results(sv.compare(pairs, a, a), len(pairs))
+    assert_results_match(got, want, "seed %d" % seed)
+    plan = sv.ComparePlan(pairs, buf.size, buf.size, device=dev)
+    got_plan = sv.decode_results(plan(a, a), len(pairs))
+    assert_results_match(got_plan, want, "plan, seed %d" % seed)
