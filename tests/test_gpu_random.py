@@ -146,3 +146,31 @@ def test_random_pair_tables_match_the_oracle(dev, seed):
     plan = sv.ComparePlan(pairs, buf.size, buf.size, device=dev)
     got_plan = sv.decode_results(plan(a, a), len(pairs))
     assert_results_match(got_plan, want, "plan, seed %d" % seed)
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_random_tile_geometries_match_the_oracle(dev, seed):
+    """Shaped outputs of random rows, columns, padded pitches and tile sizes --
+    side-by-side tile groups (with their staging ring), warp and CTA tiles,
+    ragged edges -- against the oracle's tile compare."""
+    import oracle
+    from gpu_util import assert_results_match, to_dev
+    from test_gpu_tiles import make_pair
+    rng = np.random.default_rng(9000 + seed)
+    dtype = str(rng.choice(["f32", "f16", "bf16", "i32", "i64", "u32"]))
+    sz = W.DTYPE_BYTES[dtype]
+    align = 16 // sz
+    rows = int(rng.choice([1, 3, 17, 130, 2000, 9000]))
+    cols = int(rng.choice([1, 3, 8, 40, 64, 100, 256, 520]))
+    cp = -(-(cols + int(rng.integers(0, 20))) // align) * align
+    rp = -(-(cols + int(rng.integers(0, 20))) // align) * align
+    tr = int(rng.choice([1, 2, 3, 4, 5, 7, 8, 16, 33, 128]))
+    tc = int(rng.choice([cols, 8, 16, 32, 64, 128]))
+    if tc < cols:
+        tc = -(-tc // align) * align
+    x, y = make_pair(dtype, rows, cols, cp, rp, seed=9000 + seed)
+    t = W.Tiles(dtype, rows, cols, 0, 0, cand_pitch=cp, ref_pitch=rp, tile_rows=tr, tile_cols=tc,
+                atol=1e-3, rtol=1e-3)
+    want = oracle.compare_tiles(t, x, y)
+    got = sv.decode_results(sv.compare_tiles(t, to_dev(x, dev), to_dev(y, dev)), len(want))
+    assert_results_match(got, want, "%s rows %d cols %d pitches %d/%d tile %dx%d" % (dtype, rows, cols, cp, rp, tr, tc))
