@@ -174,3 +174,43 @@ def test_random_tile_geometries_match_the_oracle(dev, seed):
     want = oracle.compare_tiles(t, x, y)
     got = sv.decode_results(sv.compare_tiles(t, to_dev(x, dev), to_dev(y, dev)), len(want))
     assert_results_match(got, want, "%s rows %d cols %d pitches %d/%d tile %dx%d" % (dtype, rows, cols, cp, rp, tr, tc))
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_random_ladders_match_the_oracle(dev, seed):
+    """Progressive ladders of 1 to 12 stages of mixed dtypes and sizes (stage
+    groups form and break on dtype changes and size limits), failing at a
+    random stage or not at all: every stage's result, the skipped ones and the
+    first failed index equal the oracle's."""
+    import oracle
+    import torch
+    from gpu_util import assert_results_match
+    rng = np.random.default_rng(13000 + seed)
+    ar = W.Arena()
+    stages, chunks = [], []
+    n_st = int(rng.integers(1, 13))
+    fail_at = int(rng.integers(0, n_st + 1))  # n_st: every stage passes
+    for i in range(n_st):
+        dt = str(rng.choice(["f32", "f32", "bf16", "i32", "i64"]))
+        n = int(rng.choice([1, 100, 4096, 50000, 1 << 20]))
+        c, r = W.random_pair_arrays(dt, n, seed=int(rng.integers(0, 1 << 30)), mismatch_frac=0.0,
+                                    nonfinite_frac=0.0)
+        if i == fail_at:
+            k = int(rng.integers(0, n))
+            sz = W.DTYPE_BYTES[dt]
+            c = c.copy()
+            c[k * sz] ^= 0x01
+            c[k * sz + sz - 1] ^= 0x10
+        sz = W.DTYPE_BYTES[dt]
+        co, ro = ar.take(n * sz), ar.take(n * sz)
+        chunks += [(co, c), (ro, r)]
+        stages.append(W.Pair(dt, n, co, ro, atol=1e-6, rtol=1e-6))
+    buf = np.zeros(ar.size, np.uint8)
+    for off, data in chunks:
+        buf[off: off + data.size] = data
+    want, want_ff = oracle.progressive(stages, buf, buf)
+    a = torch.from_numpy(buf).to(dev)
+    res, ff = sv.progressive(stages, a, a)
+    torch.cuda.synchronize()
+    assert int(ff.item()) == want_ff
+    assert_results_match(sv.decode_results(res, n_st), want, "seed %d" % seed)
